@@ -1,0 +1,130 @@
+"""Pure-Python big-integer restatement of the learning method (small cases).
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).  A second, independent
+oracle: feature rows and words are Python integers (bit k of the integer =
+feature index k; bit i of the word = output bit i), so XOR of integers is row
+addition over GF(2) (Sec. 2.2).  It is used on tiny inputs, the worked
+examples of Appendices B and C and brute-force checks, and to cross-check the
+C oracle.
+
+Training follows Sec. 2.2 steps (1)-(5) as written: reduce against the stored
+pivots, discard a zero/zero residual, report a zero-feature/nonzero-output
+residual as a contradiction, else insert with pivot = highest set feature bit
+after clearing that bit from the stored rows.  Encoding follows Sec. 2.3.
+"""
+from __future__ import annotations
+
+from typing import Dict, List, Optional, Tuple
+
+
+def phi(x: int, n: int) -> int:
+    """Feature vector [1 || x] of an n-bit feature value (index 0 = constant, Sec. 2.1)."""
+    return 1 | ((x & ((1 << n) - 1)) << 1)
+
+
+def parsed_value_features(values: List[int]) -> int:
+    """phi(x) = [1 || bits64(v_0) || ... || bits64(v_{k-1})] (Sec. 2.1), as an integer."""
+    f = 1
+    for i, v in enumerate(values):
+        f |= (v & ((1 << 64) - 1)) << (1 + 64 * i)
+    return f
+
+
+class Basis:
+    """A pivot-indexed reduced basis B[k] = (r_k, z_k) (Appendix B)."""
+
+    def __init__(self, d: int):
+        self.d = d
+        self.rows: Dict[int, Tuple[int, int]] = {}
+        self.contradictions = 0
+        self.first_contradiction: Optional[int] = None
+        self.seen = 0
+        self.trace: List[tuple] = []
+
+    @property
+    def rank(self) -> int:
+        return len(self.rows)
+
+    def reduce(self, r: int, z: int) -> Tuple[int, int, List[int]]:
+        """Step (1): XOR against stored rows whose pivot bit is set, highest first."""
+        visited = []
+        for k in sorted(self.rows, reverse=True):
+            if (r >> k) & 1:
+                rk, zk = self.rows[k]
+                r ^= rk
+                z ^= zk
+                visited.append(k)
+        return r, z, visited
+
+    def learn(self, r: int, z: int) -> str:
+        """Process one augmented row [r | z]; returns 'new', 'redundant' or 'contradiction'."""
+        idx = self.seen
+        self.seen += 1
+        r, z, visited = self.reduce(r, z)
+        if r == 0:
+            if z == 0:
+                self.trace.append(("redundant", idx, visited, r, z))
+                return "redundant"
+            self.contradictions += 1
+            if self.first_contradiction is None:
+                self.first_contradiction = idx
+            self.trace.append(("contradiction", idx, visited, r, z))
+            return "contradiction"
+        k = r.bit_length() - 1
+        for j in list(self.rows):
+            rj, zj = self.rows[j]
+            if (rj >> k) & 1:
+                self.rows[j] = (rj ^ r, zj ^ z)
+        self.rows[k] = (r, z)
+        self.trace.append(("new", idx, visited, r, z))
+        return "new"
+
+    def encode(self, q: int) -> Tuple[bool, int, int]:
+        """Sec. 2.3: returns (supported, word, residual); word is 0 when rejected."""
+        acc = 0
+        for k in sorted(self.rows, reverse=True):
+            if (q >> k) & 1:
+                rk, zk = self.rows[k]
+                q ^= rk
+                acc ^= zk
+        if q == 0:
+            return True, acc, 0
+        return False, 0, q
+
+    def solve(self) -> List[int]:
+        """W[k] = z_k for pivots, 0 elsewhere (free coordinates zero)."""
+        return [self.rows[k][1] if k in self.rows else 0 for k in range(self.d)]
+
+
+def learn_rows(d: int, rows) -> Basis:
+    B = Basis(d)
+    for r, z in rows:
+        B.learn(r, z)
+    return B
+
+
+def rank_of(vectors) -> int:
+    """Rank of a list of integer bit-vectors by elimination on the highest bit
+    over all columns (used for the consistency test rank([Phi|Y]) = rank(Phi))."""
+    piv: Dict[int, int] = {}
+    for v in vectors:
+        while v:
+            h = v.bit_length() - 1
+            if h in piv:
+                v ^= piv[h]
+            else:
+                piv[h] = v
+                break
+    return len(piv)
+
+
+def words_to_int(words) -> int:
+    """uint32 words (little-endian word order) to an integer."""
+    v = 0
+    for i, w in enumerate(words):
+        v |= int(w) << (32 * i)
+    return v
+
+
+def int_to_words(v: int, nwords: int) -> List[int]:
+    return [(v >> (32 * i)) & 0xFFFFFFFF for i in range(nwords)]
