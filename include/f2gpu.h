@@ -1,0 +1,202 @@
+/*
+ * f2gpu.h -- C ABI of libf2gpu.so: batched streaming Gaussian elimination over
+ * GF(2), affine-map extraction and batched encoding with a span check, on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * The method is the exact bit-linear encoder learner of "Learning Exact
+ * NVIDIA SASS Encoders with F2 Linear Algebra" (F2Asm):
+ *   - an encoding context receives observations (x, y), x in F2^n (feature
+ *     bits), y in F2^128 (instruction word); the feature vector is
+ *     phi(x) = [1 || x] with the affine constant at index 0 and feature bit j
+ *     at index 1+j (Sec. 2.1, parsed-value feature map), d = n + 1;
+ *   - each augmented row [phi(x) | y] is reduced against the context's
+ *     reduced basis B[k] = (r_k, z_k); zero/zero residuals are discarded, a
+ *     zero feature residual with a nonzero word residual is a contradiction,
+ *     anything else is inserted with pivot k = highest set feature index after
+ *     clearing bit k from the stored rows (Sec. 2.2, steps (1)-(5));
+ *   - the learned map is T(r_k) = z_k on S = rowspan(Phi) (Sec. 2.3);
+ *     f2_solve_affine extends it by zero on non-pivot coordinates;
+ *   - encoding reduces q = phi(x) against the basis while XOR-ing the z_k of
+ *     every row used; a zero residual proves q in S and yields T(q), otherwise
+ *     the query is rejected (Sec. 2.3, Appendix B).
+ *
+ * Conventions for every entry point:
+ *   - Pointers named *_dev are device pointers (or managed/mapped memory the
+ *     device can read); pointers named *_host are host pointers.  The caller
+ *     owns all of them; the library never frees caller memory.
+ *   - Feature words: uint32, bit j of x = bit j%32 of word j/32; a row of
+ *     context c occupies W_c = ceil(n_c/32) words; bits at positions >= n_c
+ *     are ignored.  128-bit words: four uint32 (bit i = bit i%32 of word
+ *     i/32, the little-endian numbering of Appendix C), 16-byte aligned.
+ *   - Every call is asynchronous on the caller's stream and ordered with the
+ *     caller's other work on that stream; results are valid once the stream
+ *     has been synchronized.  Calls on one store must not overlap on
+ *     different streams.
+ *   - Return value: F2_OK or an F2_ERR_* code for errors detected on the host
+ *     before anything is enqueued (nothing is enqueued on error).  Errors that
+ *     only the device can detect (bad CSR offsets, out-of-range context ids)
+ *     are recorded in the store's device status word; read it with
+ *     f2_device_status.  Contradictions and rejected queries are results,
+ *     not errors.
+ */
+#ifndef F2GPU_H
+#define F2GPU_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* f2_stream_t;
+
+typedef struct f2_store f2_store;
+
+enum f2_status {
+    F2_OK = 0,
+    F2_ERR_INVALID_ARG = 1, /* null pointer, negative size, bad flags, mismatched import */
+    F2_ERR_NBITS = 2,       /* a feature width outside [1, 1024] */
+    F2_ERR_CTX_RANGE = 3,   /* (device) an encode query named a context id outside [0, num_ctx) */
+    F2_ERR_ALIGN = 4,       /* a pointer misses its required alignment */
+    F2_ERR_OOM = 5,         /* device or host allocation failed */
+    F2_ERR_CUDA = 6,        /* a CUDA runtime call failed */
+    F2_ERR_TIMEOUT = 7,     /* (device) a bounded device-side wait gave up */
+    F2_ERR_ROWS = 8,        /* (device) CSR offsets of a context are decreasing or out of bounds;
+                               that context's rows were skipped */
+    F2_ERR_STRIDE = 9       /* (device) a query's context needs more words than x_stride_words */
+};
+
+/* Rows are complete feature vectors: no implicit constant, d = n, feature
+   bit j is index j.  Without this flag d = n + 1 and phi(x) = [1 || x]. */
+#define F2_FLAG_RAW_FEATURES 1u
+
+/* Text for a status code (static storage). */
+const char* f2_status_string(int status);
+
+/*
+ * Create a store of num_ctx contexts on the current CUDA device.
+ * n_bits_host[c] in [1, 1024] is context c's feature width n_c.  Allocates
+ * the basis (slot k of context c for k < d_c), pivot masks, ranks and
+ * contradiction records, all zeroed on `stream`.  On success *out receives
+ * the handle; on failure *out is NULL.
+ * Errors: F2_ERR_INVALID_ARG (out or n_bits_host NULL, num_ctx < 0, unknown
+ * flags), F2_ERR_NBITS, F2_ERR_OOM, F2_ERR_CUDA.
+ */
+int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
+              f2_stream_t stream);
+
+/* Release the store's device memory (synchronizes the device). NULL is a no-op. */
+void f2_destroy(f2_store* store);
+
+/* Forget everything learned (bases, ranks, contradiction records, row counts). */
+int f2_reset(f2_store* store, f2_stream_t stream);
+
+/*
+ * Host copies of the canonical layout offsets, each an array of num_ctx+1
+ * int64 (any may be NULL):
+ *   slot_off[c] = sum_{c'<c} d_c'              (128-bit slots: basis z, solve output)
+ *   xw_off[c]   = sum_{c'<c} d_c' * Wd_c'      (basis feature words, Wd = ceil(d/32))
+ *   pw_off[c]   = sum_{c'<c} Wd_c'             (pivot-mask words)
+ */
+int f2_layout(const f2_store* store, int64_t* slot_off, int64_t* xw_off, int64_t* pw_off);
+
+/* Number of contexts, and the total sizes of the canonical arrays. */
+int f2_sizes(const f2_store* store, int32_t* num_ctx, int64_t* slots, int64_t* basis_words,
+             int64_t* pivot_words);
+
+/*
+ * Learn one batch of observations (Sec. 2.2).  May be called repeatedly: each
+ * call continues every context's stream where the previous call stopped.
+ *   row_off_dev[num_ctx+1] (int64): rows of context c are the 128-bit words
+ *       y_dev[row_off[c] .. row_off[c+1]) in stream order (row_off[0] need
+ *       not be 0);
+ *   x_off_dev[num_ctx] (int64): row i of context c has its W_c feature words
+ *       at x_dev[x_off[c] + i*W_c];
+ *   y_dev: 4 uint32 per row, 16-byte aligned;
+ *   total_rows / total_x_words: sizes of y_dev (rows) and x_dev (words); a
+ *       context whose rows or words fall outside them is skipped and
+ *       F2_ERR_ROWS is recorded on the device.
+ * Per context: rank, reduced basis, pivot mask, contradiction flag (sticky),
+ * index of the first contradicting row (counted over the context's whole
+ * stream, across calls, from 0) and the number of contradicting rows.
+ * Contradicting rows are not inserted; learning continues after them.
+ * Scratch: the scheduling queue allocated by f2_create (one call at a time).
+ * Errors: F2_ERR_INVALID_ARG (NULL pointer or negative size), F2_ERR_ALIGN
+ * (y_dev not 16-byte aligned, offsets not 8-byte aligned), F2_ERR_CUDA.
+ */
+int f2_learn_batched(f2_store* store, const int64_t* row_off_dev, const uint32_t* x_dev,
+                     const int64_t* x_off_dev, const uint32_t* y_dev, int64_t total_rows,
+                     int64_t total_x_words, f2_stream_t stream);
+
+/*
+ * Copy the learned state into caller device buffers (any may be NULL):
+ *   rank_dev[num_ctx] int32; pivot_mask_dev[pivot_words] uint32 (bit k of
+ *   context c at word pw_off[c] + k/32); basis_x_dev[basis_words] uint32
+ *   (row k of context c at xw_off[c] + k*Wd_c: r_k, bit j = feature index
+ *   j); basis_z_dev[4*slots] uint32 (z_k at slot slot_off[c] + k);
+ *   contra_dev[num_ctx] uint8 (0/1); first_contra_dev[num_ctx] int64 (-1 if
+ *   none); n_contra_dev[num_ctx] uint64; rows_seen_dev[num_ctx] int64.
+ * Empty slots are zero.  The basis is in reduced echelon form: r_k has its
+ * highest set bit at k and is zero at every other pivot (Appendix B).
+ */
+int f2_get_basis(const f2_store* store, int32_t* rank_dev, uint32_t* pivot_mask_dev,
+                 uint32_t* basis_x_dev, uint32_t* basis_z_dev, uint8_t* contra_dev,
+                 int64_t* first_contra_dev, uint64_t* n_contra_dev, int64_t* rows_seen_dev,
+                 f2_stream_t stream);
+
+/*
+ * Affine solve (Sec. 2.3): W_dev[4*slots] receives, for context c and index
+ * j < d_c, the 128-bit row W[c][j] at slot slot_off[c] + j: z_j if j is a
+ * pivot, zero otherwise (free coordinates set to zero; W is unique only on
+ * the span).  Without F2_FLAG_RAW_FEATURES, b = W[c][0] and column j of A is
+ * W[c][1+j], so y = A x XOR b for every x whose phi(x) lies in the span.
+ * Errors: F2_ERR_INVALID_ARG, F2_ERR_ALIGN (W_dev not 16-byte aligned).
+ */
+int f2_solve_affine(const f2_store* store, uint32_t* W_dev, f2_stream_t stream);
+
+/*
+ * Encode Q queries (Sec. 2.3, Appendix B).  Query q names context
+ * ctx_id_dev[q]; its feature words are x_dev[q*x_stride_words ...].
+ * y_out_dev[4*q ..] receives T(phi(x)) when phi(x) is in the context's span
+ * and zero otherwise; in_span_dev[q] receives 1 (supported), 0 (rejected) or
+ * 0xFF (context id out of range -- F2_ERR_CTX_RANGE is recorded -- or the
+ * context needs more than x_stride_words words -- F2_ERR_STRIDE).
+ * Errors: F2_ERR_INVALID_ARG (Q < 0, NULL pointers, x_stride_words < 1),
+ * F2_ERR_ALIGN (y_out_dev not 16-byte aligned).
+ */
+int f2_encode_batched(const f2_store* store, int64_t Q, const int32_t* ctx_id_dev,
+                      const uint32_t* x_dev, int32_t x_stride_words, uint32_t* y_out_dev,
+                      uint8_t* in_span_dev, f2_stream_t stream);
+
+/*
+ * Synchronize `stream`, then read and clear the store's device status word:
+ * *status receives F2_OK or the first device-detected F2_ERR_* code since the
+ * last read.
+ */
+int f2_device_status(f2_store* store, int* status, f2_stream_t stream);
+
+/*
+ * Checkpoint: serialize the whole learned state into host memory.  With
+ * host_buf NULL, *size receives the number of bytes needed.  Otherwise
+ * *size must be at least that; the call synchronizes `stream`.
+ */
+int f2_store_export(const f2_store* store, void* host_buf, size_t* size, f2_stream_t stream);
+
+/* Restore a checkpoint written by f2_store_export from a store with the same
+   context count, widths and flags (F2_ERR_INVALID_ARG otherwise). */
+int f2_store_import(f2_store* store, const void* host_buf, size_t size, f2_stream_t stream);
+
+/* Scheduling knobs of f2_learn_batched (performance only, never results). */
+enum f2_option {
+    F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA */
+    F2_OPT_WARP_BASIS_BYTES = 2 /* largest basis (bytes of shared memory) handled by one warp */
+};
+int f2_set_option(f2_store* store, int option, int64_t value);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* F2GPU_H */

@@ -1,0 +1,117 @@
+// Batched encoding with a span check (Sec. 2.3, Appendix B) on sm_103a.
+//
+// One thread per query: q = phi(x) is reduced against its context's reduced
+// basis; every stored row used also XORs its z_k into a zero accumulator.
+// Because the basis is reduced, the rows to use are exactly the pivots set in
+// q itself, walked word by word.  A zero residual at the non-pivot columns
+// proves q in the span and the accumulator is the word; otherwise the query
+// is rejected and the word is zero.
+#include "f2_internal.cuh"
+
+using namespace f2;
+
+namespace {
+
+template <int WD>
+__device__ __forceinline__ bool encode_one(const StoreDev& s, const CtxDesc& cd, const uint32_t* __restrict__ xq,
+                                           uint4& acc)
+{
+    uint32_t q[WD];
+    {
+        uint32_t xin[WD];
+#pragma unroll
+        for (int v = 0; v < WD; ++v) {
+            uint32_t t = (v < cd.xw) ? __ldg(xq + v) : 0u;
+            if (v == cd.xw - 1 && (cd.n & 31)) t &= (1u << (cd.n & 31)) - 1u;
+            xin[v] = t;
+        }
+        if (s.raw) {
+#pragma unroll
+            for (int v = 0; v < WD; ++v) q[v] = xin[v];
+        } else {
+            q[0] = (xin[0] << 1) | 1u;
+#pragma unroll
+            for (int v = 1; v < WD; ++v) q[v] = (xin[v] << 1) | (xin[v - 1] >> 31);
+        }
+    }
+    acc = make_uint4(0, 0, 0, 0);
+    const uint32_t* __restrict__ P = s.pivot + cd.pw_off;
+    const uint4* __restrict__ Z = s.bz + cd.slot_off;
+    const uint32_t* __restrict__ X = s.bx + cd.xw_off;
+#pragma unroll
+    for (int w = 0; w < WD; ++w) {
+        if (w < cd.wd) {
+            const uint32_t pw = __ldg(P + w);
+            uint32_t m = q[w] & pw;
+            while (m) {
+                const int b = __ffs(m) - 1;
+                m &= m - 1;
+                const int k = 32 * w + b;
+                const uint4 z = __ldg(Z + k);
+                acc.x ^= z.x;
+                acc.y ^= z.y;
+                acc.z ^= z.z;
+                acc.w ^= z.w;
+                const uint32_t* rk = X + (int64_t)k * cd.wd;
+#pragma unroll
+                for (int v = 0; v <= w; ++v) q[v] ^= __ldg(rk + v);
+            }
+        }
+    }
+    // rows of higher pivots change non-pivot bits of lower words, so the
+    // residual is read only after every word has been processed
+    uint32_t resid = 0;
+#pragma unroll
+    for (int w = 0; w < WD; ++w)
+        if (w < cd.wd) resid |= q[w] & ~__ldg(P + w);
+    return resid == 0;
+}
+
+__global__ void __launch_bounds__(256) encode_kernel(StoreDev s, int64_t Q, const int32_t* __restrict__ ctx_id,
+                                                     const uint32_t* __restrict__ x, int stride,
+                                                     uint4* __restrict__ y, uint8_t* __restrict__ in_span)
+{
+    const int64_t step = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < Q; i += step) {
+        const int c = __ldg(ctx_id + i);
+        uint4 acc = make_uint4(0, 0, 0, 0);
+        uint8_t flag;
+        if (c < 0 || c >= s.num_ctx) {
+            record_status(s.status, F2_ERR_CTX_RANGE);
+            flag = 0xFF;
+        } else {
+            const CtxDesc cd = s.desc[c];
+            const uint32_t* xq = x + i * stride;
+            bool ok;
+            if (cd.xw > stride) {
+                record_status(s.status, F2_ERR_STRIDE);
+                flag = 0xFF;
+                ok = false;
+            } else {
+                ok = (cd.wd <= NARROW_WD) ? encode_one<NARROW_WD>(s, cd, xq, acc) : encode_one<33>(s, cd, xq, acc);
+                flag = ok ? 1 : 0;
+            }
+            if (!ok) acc = make_uint4(0, 0, 0, 0);
+        }
+        y[i] = acc;
+        in_span[i] = flag;
+    }
+}
+
+}  // namespace
+
+extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* ctx_id, const uint32_t* x,
+                                 int32_t x_stride_words, uint32_t* y_out, uint8_t* in_span, f2_stream_t stream)
+{
+    if (!st || Q < 0 || x_stride_words < 1) return F2_ERR_INVALID_ARG;
+    if (Q == 0) return F2_OK;
+    if (!ctx_id || !x || !y_out || !in_span) return F2_ERR_INVALID_ARG;
+    if (((uintptr_t)y_out % 16) != 0 || ((uintptr_t)x % 4) != 0 || ((uintptr_t)ctx_id % 4) != 0)
+        return F2_ERR_ALIGN;
+    int64_t blocks = (Q + 255) / 256;
+    const int64_t cap = (int64_t)st->num_sms * 8;
+    if (blocks > cap) blocks = cap;
+    encode_kernel<<<(int)blocks, 256, 0, (cudaStream_t)stream>>>(st->dev(), Q, ctx_id, x, x_stride_words,
+                                                                 reinterpret_cast<uint4*>(y_out), in_span);
+    return f2_cuda_status(cudaGetLastError());
+}

@@ -1,0 +1,122 @@
+// Internal definitions shared by the CUDA translation units of libf2gpu.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "f2gpu.h"
+
+namespace f2 {
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int MAX_N = 1024;          // feature bits per context
+constexpr int MAX_D = MAX_N + 1;     // row width with the affine constant
+constexpr int NARROW_WD = 9;         // widest row (32-bit words) handled by the narrow kernels
+constexpr int LEARN_WARPS = 8;       // warps per CTA of the narrow learn kernel
+constexpr int WIDE_WARPS = 8;        // warps per CTA of the wide learn kernel
+constexpr int PLAN_BUCKETS = 48;     // log2(work) buckets for longest-first ordering
+
+// Scheduling counters written by the plan kernel, read by the learn kernels.
+enum Counter {
+    CNT_HEAD_CTA = 0,  // next item of the CTA queue (narrow contexts, one CTA each)
+    CNT_HEAD_WIDE = 1, // next item of the wide queue
+    CNT_HEAD_WARP = 2, // next item of the warp queue
+    CNT_BEGIN = 3,     // 3 + class: first queue slot of each class
+    CNT_COUNT = 6,     // 6 + class: number of contexts of each class
+    CNT_TOTAL = 9
+};
+enum Class { CLS_CTA = 0, CLS_WIDE = 1, CLS_WARP = 2 };
+
+// Per-context descriptor (device copy built at store creation).
+struct CtxDesc {
+    int32_t n;        // feature bits as supplied
+    int32_t d;        // row width (n + 1, or n for raw feature rows)
+    int32_t wd;       // 32-bit words of a feature row: ceil(d / 32)
+    int32_t xw;       // 32-bit words of a supplied feature vector: ceil(n / 32)
+    int64_t slot_off; // first 128-bit slot (basis z, solve output)
+    int64_t xw_off;   // first basis feature word (d * wd words)
+    int64_t pw_off;   // first pivot-mask word (wd words)
+    int64_t pad;
+};
+
+// Device view of a store.
+struct StoreDev {
+    const CtxDesc* desc;
+    int32_t* rank;
+    uint8_t* contra;
+    long long* first_contra;
+    unsigned long long* n_contra;
+    long long* rows_seen;
+    uint32_t* pivot;
+    uint32_t* bx;
+    uint4* bz;
+    int* status;
+    int32_t num_ctx;
+    uint32_t raw;
+};
+
+// Shared-memory row stride (32-bit words) of a basis slot: the 128-bit z
+// first, then the wd feature words, padded to 16 bytes.
+__host__ __device__ constexpr int row_stride(int wd) { return 4 * ((4 + wd + 3) / 4); }
+
+__device__ __forceinline__ void record_status(int* status, int code)
+{
+    atomicCAS(status, 0, code);
+}
+
+}  // namespace f2
+
+struct f2_store {
+    int32_t num_ctx;
+    uint32_t flags;
+    int device;
+    int num_sms;
+    int32_t max_wd;
+    int32_t max_d;
+    int32_t n_wide;         // contexts with wd > NARROW_WD
+    int64_t slots;
+    int64_t basis_words;
+    int64_t pivot_words;
+    int64_t heavy_rows;
+    int64_t warp_basis_bytes;
+    std::vector<int32_t> n_bits;
+    std::vector<int64_t> slot_off, xw_off, pw_off;
+    // device memory
+    f2::CtxDesc* desc;
+    int32_t* rank;
+    uint8_t* contra;
+    long long* first_contra;
+    unsigned long long* n_contra;
+    long long* rows_seen;
+    uint32_t* pivot;
+    uint32_t* bx;
+    uint4* bz;
+    int* status;
+    // scheduling scratch of f2_learn_batched
+    int32_t* queue;
+    int32_t* keybuf;
+    int* counters;
+
+    f2::StoreDev dev() const
+    {
+        f2::StoreDev s;
+        s.desc = desc;
+        s.rank = rank;
+        s.contra = contra;
+        s.first_contra = first_contra;
+        s.n_contra = n_contra;
+        s.rows_seen = rows_seen;
+        s.pivot = pivot;
+        s.bx = bx;
+        s.bz = bz;
+        s.status = status;
+        s.num_ctx = num_ctx;
+        s.raw = (flags & F2_FLAG_RAW_FEATURES) ? 1u : 0u;
+        return s;
+    }
+};
+
+// Host helpers (store.cu).
+int f2_cuda_status(cudaError_t e);

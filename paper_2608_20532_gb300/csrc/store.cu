@@ -1,0 +1,363 @@
+// Store management, layout queries, checkpointing and the affine solve.
+#include <stdlib.h>
+#include <string.h>
+
+#include <new>
+
+#include "f2_internal.cuh"
+
+using namespace f2;
+
+int f2_cuda_status(cudaError_t e)
+{
+    if (e == cudaSuccess) return F2_OK;
+    if (e == cudaErrorMemoryAllocation) return F2_ERR_OOM;
+    return F2_ERR_CUDA;
+}
+
+static inline bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+extern "C" const char* f2_status_string(int status)
+{
+    switch (status) {
+    case F2_OK: return "ok";
+    case F2_ERR_INVALID_ARG: return "invalid argument";
+    case F2_ERR_NBITS: return "feature width outside [1, 1024]";
+    case F2_ERR_CTX_RANGE: return "context id out of range";
+    case F2_ERR_ALIGN: return "pointer misaligned";
+    case F2_ERR_OOM: return "out of memory";
+    case F2_ERR_CUDA: return "CUDA runtime error";
+    case F2_ERR_TIMEOUT: return "bounded device wait gave up";
+    case F2_ERR_ROWS: return "CSR offsets decreasing or out of bounds";
+    case F2_ERR_STRIDE: return "query stride narrower than the context's feature words";
+    default: return "unknown status";
+    }
+}
+
+static void free_store(f2_store* s)
+{
+    if (!s) return;
+    void* ptrs[] = {s->desc, s->rank, s->contra, s->first_contra, s->n_contra, s->rows_seen, s->pivot,
+                    s->bx, s->bz, s->status, s->queue, s->keybuf, s->counters};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    delete s;
+}
+
+static cudaError_t zero_state(f2_store* s, cudaStream_t st)
+{
+    cudaError_t e = cudaSuccess;
+    auto z = [&](void* p, size_t bytes) {
+        if (e == cudaSuccess && bytes) e = cudaMemsetAsync(p, 0, bytes, st);
+    };
+    z(s->rank, sizeof(int32_t) * (size_t)s->num_ctx);
+    z(s->contra, (size_t)s->num_ctx);
+    z(s->n_contra, sizeof(unsigned long long) * (size_t)s->num_ctx);
+    z(s->rows_seen, sizeof(long long) * (size_t)s->num_ctx);
+    z(s->pivot, sizeof(uint32_t) * (size_t)s->pivot_words);
+    z(s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
+    z(s->bz, sizeof(uint4) * (size_t)s->slots);
+    if (e == cudaSuccess && s->num_ctx)  // first_contra = -1 (all bytes 0xff)
+        e = cudaMemsetAsync(s->first_contra, 0xff, sizeof(long long) * (size_t)s->num_ctx, st);
+    z(s->status, sizeof(int));
+    return e;
+}
+
+extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
+                         f2_stream_t stream)
+{
+    if (!out) return F2_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (num_ctx < 0 || (num_ctx > 0 && !n_bits_host) || (flags & ~F2_FLAG_RAW_FEATURES))
+        return F2_ERR_INVALID_ARG;
+    for (int32_t c = 0; c < num_ctx; ++c)
+        if (n_bits_host[c] < 1 || n_bits_host[c] > MAX_N) return F2_ERR_NBITS;
+    f2_store* s = new (std::nothrow) f2_store();
+    if (!s) return F2_ERR_OOM;
+    s->num_ctx = num_ctx;
+    s->flags = flags;
+    s->heavy_rows = 4096;
+    s->warp_basis_bytes = 8192;
+    if (cudaGetDevice(&s->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
+        delete s;
+        return F2_ERR_CUDA;
+    }
+    const bool raw = (flags & F2_FLAG_RAW_FEATURES) != 0;
+    std::vector<CtxDesc> desc((size_t)num_ctx);
+    s->n_bits.assign(n_bits_host, n_bits_host + num_ctx);
+    s->slot_off.assign((size_t)num_ctx + 1, 0);
+    s->xw_off.assign((size_t)num_ctx + 1, 0);
+    s->pw_off.assign((size_t)num_ctx + 1, 0);
+    for (int32_t c = 0; c < num_ctx; ++c) {
+        CtxDesc& cd = desc[(size_t)c];
+        cd.n = n_bits_host[c];
+        cd.d = raw ? cd.n : cd.n + 1;
+        cd.wd = (cd.d + 31) / 32;
+        cd.xw = (cd.n + 31) / 32;
+        cd.slot_off = s->slot_off[(size_t)c];
+        cd.xw_off = s->xw_off[(size_t)c];
+        cd.pw_off = s->pw_off[(size_t)c];
+        cd.pad = 0;
+        s->slot_off[(size_t)c + 1] = cd.slot_off + cd.d;
+        s->xw_off[(size_t)c + 1] = cd.xw_off + (int64_t)cd.d * cd.wd;
+        s->pw_off[(size_t)c + 1] = cd.pw_off + cd.wd;
+        if (cd.wd > s->max_wd) s->max_wd = cd.wd;
+        if (cd.d > s->max_d) s->max_d = cd.d;
+        if (cd.wd > NARROW_WD) s->n_wide++;
+    }
+    s->slots = s->slot_off[(size_t)num_ctx];
+    s->basis_words = s->xw_off[(size_t)num_ctx];
+    s->pivot_words = s->pw_off[(size_t)num_ctx];
+
+    cudaError_t e = cudaSuccess;
+    auto alloc = [&](void** p, size_t bytes) {
+        if (e == cudaSuccess) e = cudaMalloc(p, bytes ? bytes : 16);
+    };
+    const size_t C = (size_t)(num_ctx > 0 ? num_ctx : 1);
+    alloc((void**)&s->desc, sizeof(CtxDesc) * C);
+    alloc((void**)&s->rank, sizeof(int32_t) * C);
+    alloc((void**)&s->contra, C);
+    alloc((void**)&s->first_contra, sizeof(long long) * C);
+    alloc((void**)&s->n_contra, sizeof(unsigned long long) * C);
+    alloc((void**)&s->rows_seen, sizeof(long long) * C);
+    alloc((void**)&s->pivot, sizeof(uint32_t) * (size_t)s->pivot_words);
+    alloc((void**)&s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
+    alloc((void**)&s->bz, sizeof(uint4) * (size_t)s->slots);
+    alloc((void**)&s->status, sizeof(int));
+    alloc((void**)&s->queue, sizeof(int32_t) * C);
+    alloc((void**)&s->keybuf, sizeof(int32_t) * C);
+    alloc((void**)&s->counters, sizeof(int) * 16);
+    cudaStream_t st = (cudaStream_t)stream;
+    if (e == cudaSuccess && num_ctx)
+        e = cudaMemcpyAsync(s->desc, desc.data(), sizeof(CtxDesc) * (size_t)num_ctx,
+                            cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = zero_state(s, st);
+    // the host vector `desc` must outlive the copy
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        int code = f2_cuda_status(e);
+        free_store(s);
+        return code;
+    }
+    *out = s;
+    return F2_OK;
+}
+
+extern "C" void f2_destroy(f2_store* store)
+{
+    if (!store) return;
+    cudaDeviceSynchronize();
+    free_store(store);
+}
+
+extern "C" int f2_reset(f2_store* s, f2_stream_t stream)
+{
+    if (!s) return F2_ERR_INVALID_ARG;
+    return f2_cuda_status(zero_state(s, (cudaStream_t)stream));
+}
+
+extern "C" int f2_layout(const f2_store* s, int64_t* slot_off, int64_t* xw_off, int64_t* pw_off)
+{
+    if (!s) return F2_ERR_INVALID_ARG;
+    const size_t n = (size_t)s->num_ctx + 1;
+    if (slot_off) memcpy(slot_off, s->slot_off.data(), n * sizeof(int64_t));
+    if (xw_off) memcpy(xw_off, s->xw_off.data(), n * sizeof(int64_t));
+    if (pw_off) memcpy(pw_off, s->pw_off.data(), n * sizeof(int64_t));
+    return F2_OK;
+}
+
+extern "C" int f2_sizes(const f2_store* s, int32_t* num_ctx, int64_t* slots, int64_t* basis_words,
+                        int64_t* pivot_words)
+{
+    if (!s) return F2_ERR_INVALID_ARG;
+    if (num_ctx) *num_ctx = s->num_ctx;
+    if (slots) *slots = s->slots;
+    if (basis_words) *basis_words = s->basis_words;
+    if (pivot_words) *pivot_words = s->pivot_words;
+    return F2_OK;
+}
+
+extern "C" int f2_get_basis(const f2_store* s, int32_t* rank, uint32_t* pivot_mask, uint32_t* basis_x,
+                            uint32_t* basis_z, uint8_t* contra, int64_t* first_contra, uint64_t* n_contra,
+                            int64_t* rows_seen, f2_stream_t stream)
+{
+    if (!s) return F2_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t C = (size_t)s->num_ctx;
+    cudaError_t e = cudaSuccess;
+    auto cp = [&](void* dst, const void* src, size_t bytes) {
+        if (e == cudaSuccess && dst && bytes) e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st);
+    };
+    cp(rank, s->rank, sizeof(int32_t) * C);
+    cp(pivot_mask, s->pivot, sizeof(uint32_t) * (size_t)s->pivot_words);
+    cp(basis_x, s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
+    cp(basis_z, s->bz, sizeof(uint4) * (size_t)s->slots);
+    cp(contra, s->contra, C);
+    cp(first_contra, s->first_contra, sizeof(int64_t) * C);
+    cp(n_contra, s->n_contra, sizeof(uint64_t) * C);
+    cp(rows_seen, s->rows_seen, sizeof(int64_t) * C);
+    return f2_cuda_status(e);
+}
+
+// ------------------------------------------------------------ affine solve
+//
+// W[c][j] = z_j for a pivot j, 0 otherwise (the learned map T of Sec. 2.3
+// extended by zero on the free coordinates).  One warp per context, lanes
+// over slots: coalesced 16-byte stores.
+__global__ void __launch_bounds__(256) solve_kernel(StoreDev s, uint4* __restrict__ W)
+{
+    const int lane = threadIdx.x & 31;
+    const int warps = (gridDim.x * blockDim.x) >> 5;
+    for (int c = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; c < s.num_ctx; c += warps) {
+        const CtxDesc cd = s.desc[c];
+        const uint32_t* P = s.pivot + cd.pw_off;
+        for (int j = lane; j < cd.d; j += 32) {
+            const bool piv = (__ldg(P + (j >> 5)) >> (j & 31)) & 1u;
+            W[cd.slot_off + j] = piv ? __ldg(s.bz + cd.slot_off + j) : make_uint4(0, 0, 0, 0);
+        }
+    }
+}
+
+extern "C" int f2_solve_affine(const f2_store* s, uint32_t* W, f2_stream_t stream)
+{
+    if (!s || (!W && s->slots)) return F2_ERR_INVALID_ARG;
+    if (!aligned(W, 16)) return F2_ERR_ALIGN;
+    if (s->num_ctx == 0) return F2_OK;
+    const int threads = 256;
+    int blocks = (int)((s->num_ctx + 7) / 8);
+    const int cap = s->num_sms * 8;
+    if (blocks > cap) blocks = cap;
+    solve_kernel<<<blocks, threads, 0, (cudaStream_t)stream>>>(s->dev(), reinterpret_cast<uint4*>(W));
+    return f2_cuda_status(cudaGetLastError());
+}
+
+extern "C" int f2_device_status(f2_store* s, int* status, f2_stream_t stream)
+{
+    if (!s || !status) return F2_ERR_INVALID_ARG;
+    cudaStream_t st = (cudaStream_t)stream;
+    int v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, s->status, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->status, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    *status = v;
+    return F2_OK;
+}
+
+// ------------------------------------------------------------ checkpoints
+
+namespace {
+struct CkptHeader {
+    char magic[8];
+    int32_t version;
+    int32_t num_ctx;
+    uint32_t flags;
+    int32_t pad;
+    int64_t slots, basis_words, pivot_words;
+};
+
+size_t ckpt_size(const f2_store* s)
+{
+    const size_t C = (size_t)s->num_ctx;
+    return sizeof(CkptHeader) + C * sizeof(int32_t) /* n_bits */ + C * sizeof(int32_t) /* rank */ +
+           C /* contra */ + C * 8 * 3 /* first, n_contra, rows_seen */ +
+           (size_t)s->pivot_words * 4 + (size_t)s->basis_words * 4 + (size_t)s->slots * 16;
+}
+}  // namespace
+
+extern "C" int f2_store_export(const f2_store* s, void* host_buf, size_t* size, f2_stream_t stream)
+{
+    if (!s || !size) return F2_ERR_INVALID_ARG;
+    const size_t need = ckpt_size(s);
+    if (!host_buf) {
+        *size = need;
+        return F2_OK;
+    }
+    if (*size < need) return F2_ERR_INVALID_ARG;
+    *size = need;
+    cudaStream_t st = (cudaStream_t)stream;
+    char* p = (char*)host_buf;
+    CkptHeader h;
+    memset(&h, 0, sizeof h);
+    memcpy(h.magic, "F2GPUCK1", 8);
+    h.version = 1;
+    h.num_ctx = s->num_ctx;
+    h.flags = s->flags;
+    h.slots = s->slots;
+    h.basis_words = s->basis_words;
+    h.pivot_words = s->pivot_words;
+    memcpy(p, &h, sizeof h);
+    p += sizeof h;
+    const size_t C = (size_t)s->num_ctx;
+    memcpy(p, s->n_bits.data(), C * 4);
+    p += C * 4;
+    cudaError_t e = cudaSuccess;
+    auto d2h = [&](const void* src, size_t bytes) {
+        if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(p, src, bytes, cudaMemcpyDeviceToHost, st);
+        p += bytes;
+    };
+    d2h(s->rank, C * 4);
+    d2h(s->contra, C);
+    d2h(s->first_contra, C * 8);
+    d2h(s->n_contra, C * 8);
+    d2h(s->rows_seen, C * 8);
+    d2h(s->pivot, (size_t)s->pivot_words * 4);
+    d2h(s->bx, (size_t)s->basis_words * 4);
+    d2h(s->bz, (size_t)s->slots * 16);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return f2_cuda_status(e);
+}
+
+extern "C" int f2_store_import(f2_store* s, const void* host_buf, size_t size, f2_stream_t stream)
+{
+    if (!s || !host_buf) return F2_ERR_INVALID_ARG;
+    const size_t need = ckpt_size(s);
+    if (size < need) return F2_ERR_INVALID_ARG;
+    const char* p = (const char*)host_buf;
+    CkptHeader h;
+    memcpy(&h, p, sizeof h);
+    if (memcmp(h.magic, "F2GPUCK1", 8) != 0 || h.version != 1 || h.num_ctx != s->num_ctx ||
+        h.flags != s->flags || h.slots != s->slots || h.basis_words != s->basis_words ||
+        h.pivot_words != s->pivot_words)
+        return F2_ERR_INVALID_ARG;
+    p += sizeof h;
+    const size_t C = (size_t)s->num_ctx;
+    if (memcmp(p, s->n_bits.data(), C * 4) != 0) return F2_ERR_INVALID_ARG;
+    p += C * 4;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaSuccess;
+    auto h2d = [&](void* dst, size_t bytes) {
+        if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(dst, p, bytes, cudaMemcpyHostToDevice, st);
+        p += bytes;
+    };
+    h2d(s->rank, C * 4);
+    h2d(s->contra, C);
+    h2d(s->first_contra, C * 8);
+    h2d(s->n_contra, C * 8);
+    h2d(s->rows_seen, C * 8);
+    h2d(s->pivot, (size_t)s->pivot_words * 4);
+    h2d(s->bx, (size_t)s->basis_words * 4);
+    h2d(s->bz, (size_t)s->slots * 16);
+    // the caller's buffer must stay valid until the copies complete
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return f2_cuda_status(e);
+}
+
+extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
+{
+    if (!s) return F2_ERR_INVALID_ARG;
+    switch (option) {
+    case F2_OPT_HEAVY_ROWS:
+        if (value < 1) return F2_ERR_INVALID_ARG;
+        s->heavy_rows = value;
+        return F2_OK;
+    case F2_OPT_WARP_BASIS_BYTES:
+        if (value < 0 || value > 24576) return F2_ERR_INVALID_ARG;
+        s->warp_basis_bytes = (value / 16) * 16;
+        return F2_OK;
+    default:
+        return F2_ERR_INVALID_ARG;
+    }
+}

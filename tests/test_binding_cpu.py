@@ -1,0 +1,59 @@
+"""The C ABI library builds for sm_103a and exports every entry point that
+include/f2gpu.h declares (no compute calls: no GPU needed)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    with open(os.path.join(ROOT, "include", "f2gpu.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(f2_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def libpath():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2608_20532_gb300 import binding
+
+    return binding.library_path()
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for required in ("f2_create", "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched",
+                     "f2_store_export", "f2_store_import", "f2_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(libpath):
+    lib = ctypes.CDLL(libpath)
+    for name in _declared():
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", libpath], capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\bT (f2_[a-z_]+)", out))
+    assert set(_declared()) <= exported
+
+
+def test_binding_covers_every_symbol(libpath):
+    from paper_2608_20532_gb300 import binding
+
+    assert set(binding.EXPORTS) == set(_declared())
+    lib = binding.load_library()
+    assert lib.f2_status_string(0).decode() == "ok"
+    assert "out of range" in lib.f2_status_string(3).decode()
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    from paper_2608_20532_gb300 import binding
+
+    with pytest.raises(RuntimeError):
+        binding.load_library(str(tmp_path / "nope.so"))
