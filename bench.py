@@ -1,0 +1,621 @@
+#!/usr/bin/env python3
+"""Throughput of the GF(2) encoder-learning hot path on GB300.
+
+Default workload (one "step"): learn the joint-Blackwell-scale synthetic
+store -- 77,926 contexts, n log-normal (median 64) in [16, 256], ~80M
+observations with 85% duplicates and 49,566 two-variant-stream contexts --
+from scratch (reset + f2_learn_batched), solve every affine map
+(f2_solve_affine), then encode 10M Zipf(1.1) queries with the span check
+(f2_encode_batched).  Inputs are resident in HBM when the timed region starts
+and are larger than L2 (2+ GB), so no L2 flush is needed.
+
+Prints one JSON line.  ``value`` = observations eliminated per second over
+the whole step; the encode throughput and per-phase times are reported
+beside it.  ``--impl reference`` times the plain CPU oracle on the host
+cores on a bounded sample of the same workload.
+
+Other workloads: ``--config 1|2|5`` (learn + solve, plus encode for 1).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "GF(2) rows eliminated/sec and words encoded/sec at 1 GB300; % HBM/INT roofline"
+HBM_FALLBACK_GBS = 6800.0
+SMS = 152
+INT_LANES_PER_SM = 64      # 32-bit logic lanes per SM per clock (4 SMSPs x 16)
+SM_MAX_MHZ_FALLBACK = 2070.0
+
+
+# ----------------------------------------------------------------- helpers
+
+def measured_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "sm_max_mhz": float(d.get("sm_max_mhz", SM_MAX_MHZ_FALLBACK)),
+                "source": "measured (MEASURED_PEAKS.json)"}
+    return {"hbm_gbs": HBM_FALLBACK_GBS, "sm_max_mhz": SM_MAX_MHZ_FALLBACK, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-i",
+                 str(gpu_index), "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.samples.append((time.time(), parts))
+
+    def stop(self, t0: float, t1: float) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        inside = [p for t, p in self.samples if t0 <= t <= t1]
+        if not inside and self.samples:  # region shorter than the sampling period: nearest samples
+            inside = [p for t, p in sorted(self.samples, key=lambda s: abs(s[0] - (t0 + t1) / 2))[:2]]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+
+        mhz = [num(p[1]) for p in inside if num(p[1]) is not None]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for p in inside:
+            for name, v in zip(names, p[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(mhz) if mhz else None, "sm_max_mhz": num(inside[0][2]),
+                "power_w_max": max((num(p[3]) or 0.0) for p in inside), "reasons": sorted(reasons),
+                "samples": len(inside)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def workload_for(cfg_id: int, rank: int, query_count=None):
+    from paper_2608_20532_gb300 import workloads as W
+
+    cfg = dict(W.CONFIGS[cfg_id])
+    seed = W.seed_for(cfg_id) + 1000 * rank
+    return W.generate(cfg, seed, name=f"config{cfg_id}", query_count=query_count)
+
+
+def describe(cfg_id: int, wl) -> dict:
+    d = {"workload": {1: "config-1 parity case: 256 contexts, n=48, 260 rows each, 100 queries/context",
+                      2: "4,096 contexts, n in [32,128], ~2.6M rows",
+                      3: "joint-Blackwell-scale learn (77,926 contexts, ~80M rows, 85% duplicates) + 10M Zipf(1.1) encode queries",
+                      5: "64 contexts, n=1024, 2^20 rows each in 16 incremental 65,536-row batches"}[cfg_id],
+         "contexts": wl.num_ctx, "rows": wl.total_rows, "n_median": float(np.median(wl.n_bits)),
+         "queries": int(len(wl.queries.ctx_id)) if wl.queries is not None else 0,
+         "input_bytes": int(wl.x.nbytes + wl.y.nbytes),
+         "l2": "inputs larger than L2 (no flush)" if wl.x.nbytes + wl.y.nbytes > 129e6 else "L2 flushed between steps"}
+    return d
+
+
+def algorithmic_bytes_learn(wl) -> int:
+    """Packed x (ceil(n/8) bytes, constant implicit) + 16 bytes of y per row."""
+    return int((wl.rows * ((wl.n_bits.astype(np.int64) + 7) // 8 + 16)).sum())
+
+
+def algorithmic_bytes_encode(wl, basis_bytes_touched: int) -> int:
+    q = wl.queries
+    n = wl.n_bits.astype(np.int64)[q.ctx_id]
+    return int((4 + (n + 7) // 8 + 16 + 1).sum()) + int(basis_bytes_touched)
+
+
+def _popcount(t):
+    t = t - ((t >> 1) & 0x55555555)
+    t = (t & 0x33333333) + ((t >> 2) & 0x33333333)
+    t = (t + (t >> 4)) & 0x0F0F0F0F
+    return ((t * 0x01010101) & 0xFFFFFFFF) >> 24
+
+
+def _q_words(xw_rows, g, dev):
+    """[1 || x] words (int64 holding 32-bit values) of rows with g x-words."""
+    import torch
+
+    X = xw_rows & 0xFFFFFFFF
+    Q = torch.zeros((X.shape[0], g + 1), dtype=torch.int64, device=dev)
+    Q[:, :g] = (X << 1) & 0xFFFFFFFF
+    Q[:, 1:] |= X >> 31
+    Q[:, 0] |= 1
+    return Q
+
+
+def algorithmic_ops(wl, pivot_words, pw_off, dev, queries=False) -> int:
+    """Sum over rows (or queries) of |q AND P| * (wd + 4): the 32-bit word
+    XORs of step (1) against the final reduced basis."""
+    import torch
+
+    n = wl.n_bits.astype(np.int64)
+    xw = (n + 31) // 32
+    wd = (n + 1 + 31) // 32
+    wdmax = int(wd.max())
+    C = wl.num_ctx
+    P = np.zeros((C, wdmax + 1), np.int64)
+    for c_w in range(wdmax):
+        has = wd > c_w
+        P[has, c_w] = pivot_words[pw_off[:-1][has] + c_w].astype(np.int64) & 0xFFFFFFFF
+    Pt = torch.from_numpy(P).to(dev)
+    total = 0
+    if queries:
+        q = wl.queries
+        ctx = torch.from_numpy(q.ctx_id.astype(np.int64)).to(dev)
+        X = torch.from_numpy(q.x.view(np.int32).astype(np.int64)).to(dev)
+        wd4 = torch.from_numpy(wd + 4).to(dev)
+        for g in np.unique(xw):
+            sel = torch.from_numpy(np.flatnonzero(xw[q.ctx_id] == g)).to(dev)
+            if sel.numel() == 0:
+                continue
+            Q = _q_words(X[sel][:, :g], int(g), dev)
+            cnt = _popcount(Q & Pt[ctx[sel]][:, :g + 1]).sum(dim=1)
+            total += int((cnt * wd4[ctx[sel]]).sum())
+        return total
+    xs = torch.from_numpy(wl.x.view(np.int32).astype(np.int64)).to(dev)
+    for g in np.unique(xw):
+        cs = np.flatnonzero(xw == g)
+        for chunk in np.array_split(cs, max(1, len(cs) // 8000)):
+            rows = wl.rows[chunk]
+            R = int(rows.sum())
+            if R == 0:
+                continue
+            starts = np.repeat(wl.x_off[chunk], rows) + (np.arange(R) - np.repeat(np.cumsum(rows) - rows, rows)) * g
+            idx = torch.from_numpy(starts).to(dev)[:, None] + torch.arange(int(g), device=dev)[None, :]
+            Q = _q_words(xs[idx], int(g), dev)
+            ctx = torch.from_numpy(np.repeat(chunk, rows)).to(dev)
+            cnt = _popcount(Q & Pt[ctx][:, :g + 1]).sum(dim=1)
+            total += int((cnt * torch.from_numpy(wd + 4).to(dev)[ctx]).sum())
+    return total
+
+
+# --------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+
+    if rank == 0:
+        __graft_entry__.build()
+    if world > 1:
+        torch.distributed.barrier()
+    from paper_2608_20532_gb300 import binding
+
+    binding.load_library()
+    cfg_id = args.config
+    wl = workload_for(cfg_id, rank)
+    t = lambda a: binding.to_device(a, dev)
+    x_t, y_t = t(wl.x), t(wl.y)
+    batches = [(t(ro), t(xo)) for ro, xo in wl.batches]
+    has_q = wl.queries is not None
+    if has_q:
+        ctx_t, qx_t = t(wl.queries.ctx_id), t(wl.queries.x)
+        Q = int(ctx_t.numel())
+        y_out = torch.empty((Q, 4), dtype=torch.int32, device=dev)
+        span = torch.empty(Q, dtype=torch.uint8, device=dev)
+    store = binding.Store(wl.n_bits, device=dev)
+    W_out = torch.empty((int(store.slot_off[-1]), 4), dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    nev = 4
+
+    def step(evs=None):
+        if evs is not None:
+            evs[0].record(stream)
+        store.reset()
+        for ro, xo in batches:
+            store.learn(ro, x_t, xo, y_t)
+        if evs is not None:
+            evs[1].record(stream)
+        store.solve(out=W_out)
+        if evs is not None:
+            evs[2].record(stream)
+        if has_q:
+            store.encode(ctx_t, qx_t, y_out, span)
+        if evs is not None:
+            evs[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = store.device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after warm-up")
+
+    K = args.steps
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(nev)] for _ in range(K)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t0 = time.time()
+    start.record(stream)
+    for k in range(K):
+        step(events[k])
+    end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop(t0, t1)
+    total_ms = start.elapsed_time(end)
+    learn_ms = [e[0].elapsed_time(e[1]) for e in events]
+    solve_ms = [e[1].elapsed_time(e[2]) for e in events]
+    enc_ms = [e[2].elapsed_time(e[3]) for e in events]
+    if world > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_step = total_ms / K
+
+    # results (for accounting) and a sanity check of the final state
+    b = store.basis()
+    torch.cuda.synchronize()
+    pivots = binding.to_numpy(b["pivot_mask"]).view(np.uint32)
+    contra = int(binding.to_numpy(b["contra"]).sum())
+    rows_total = wl.total_rows * world
+    value = rows_total / (ms_step / 1e3)
+
+    # ---- e2e through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int32) if a.dtype == np.uint32 else a)).pin_memory()
+        hx, hy = pin(wl.x), pin(wl.y)
+        hb = [(pin(ro), pin(xo)) for ro, xo in wl.batches]
+        h_in = [hx, hy] + [a for pair in hb for a in pair]
+        d_in = [x_t, y_t] + [a for pair in batches for a in pair]
+        if has_q:
+            h_in += [pin(wl.queries.ctx_id), pin(wl.queries.x)]
+            d_in += [ctx_t, qx_t]
+        outs = {k: v for k, v in store.basis().items()}
+        outs["W"] = W_out
+        if has_q:
+            outs["y"] = y_out
+            outs["span"] = span
+        h_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in outs.items()}
+        bi = sum(h.numel() * h.element_size() for h in h_in)
+        bo = sum(h.numel() * h.element_size() for h in h_out.values())
+
+        def e2e_step():
+            for h, d in zip(h_in, d_in):
+                d.copy_(h, non_blocking=True)
+            step()
+            bb = store.basis()
+            for k in ("rank", "pivot_mask", "basis_x", "basis_z", "contra", "first_contra", "n_contra",
+                      "rows_seen"):
+                h_out[k].copy_(bb[k], non_blocking=True)
+            h_out["W"].copy_(W_out, non_blocking=True)
+            if has_q:
+                h_out["y"].copy_(y_out, non_blocking=True)
+                h_out["span"].copy_(span, non_blocking=True)
+
+        Ke = max(1, min(K, args.e2e_steps))
+        for _ in range(min(2, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = s0.elapsed_time(s1) / Ke
+        if world > 1:
+            tt = torch.tensor([e_ms], device=dev)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        e2e = {"value": rows_total / (e_ms / 1e3), "unit": "rows/s", "ms_per_step": e_ms, "steps": Ke,
+               "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo)}
+
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    peaks = measured_peaks()
+    # ALU peak: derived from unit counts and the max clock; the probe checks it
+    alu_peak = SMS * INT_LANES_PER_SM * peaks["sm_max_mhz"] * 1e6
+    probe = None
+    if not args.no_probe:
+        out = torch.zeros(4096, dtype=torch.int32, device=dev)
+        iters = 4096
+        blocks = SMS * 8
+        binding.peak_lop3(blocks, 64, out)
+        torch.cuda.synchronize()
+        p0 = torch.cuda.Event(enable_timing=True)
+        p1 = torch.cuda.Event(enable_timing=True)
+        p0.record(stream)
+        nops = binding.peak_lop3(blocks, iters, out)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        probe = nops / (p0.elapsed_time(p1) / 1e3)
+
+    learn_mean = statistics.mean(learn_ms) / 1e3
+    bytes_learn = algorithmic_bytes_learn(wl)
+    ops_learn = algorithmic_ops(wl, pivots, store.pw_off, dev)
+    hbm_peak = peaks["hbm_gbs"] * 1e9
+    t_hbm, t_alu = bytes_learn / hbm_peak, ops_learn / alu_peak
+    learn_bound = "hbm" if t_hbm >= t_alu else "alu"
+    rl_learn = {
+        "kernel": "f2_learn_batched (plan_kernel + learn_narrow_kernel)",
+        "hbm": {"achieved": bytes_learn / learn_mean / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": (bytes_learn / learn_mean) / hbm_peak, "bytes_per_launch": bytes_learn},
+        "alu": {"achieved": ops_learn / learn_mean / 1e12, "peak": alu_peak / 1e12, "unit": "Tops/s",
+                "frac": (ops_learn / learn_mean) / alu_peak, "ops_per_launch": ops_learn,
+                "peak_probe_lop3": (probe / 1e12) if probe else None},
+    }
+    traffic = profile_traffic("learn_narrow_kernel")
+    dom = rl_learn[learn_bound]
+    roofline = {"bound": learn_bound, "achieved": dom["achieved"], "peak": dom["peak"], "unit": dom["unit"],
+                "frac": dom["frac"], "traffic": traffic,
+                "peak_source": peaks["source"] if learn_bound == "hbm" else
+                "derived: 152 SMs x 64 INT32 lanes x max SM clock"}
+    result = {
+        "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u32", "data": "synthetic (seeded planted affine maps)",
+        "config": dict(describe(cfg_id, wl), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
+        "phases_ms": {"learn": statistics.mean(learn_ms), "solve": statistics.mean(solve_ms),
+                      "encode": statistics.mean(enc_ms)},
+        "learn_rows_per_s": wl.total_rows / learn_mean,
+        "roofline": roofline,
+        "roofline_learn": rl_learn,
+        "clocks": clocks,
+        "gpu_launches": K * (len(wl.batches) * (1 + int(store_has_narrow(wl)) + int(store_has_wide(wl)))
+                             + 1 + int(has_q)),
+        "contradiction_contexts": contra,
+    }
+    if has_q:
+        enc_mean = statistics.mean(enc_ms) / 1e3
+        span_np = binding.to_numpy(span)
+        ops_enc = algorithmic_ops(wl, pivots, store.pw_off, dev, queries=True)
+        bytes_enc = algorithmic_bytes_encode(wl, basis_bytes_touched(wl, store))
+        result["encode_words_per_s"] = Q / enc_mean
+        result["encode_in_span_frac"] = float((span_np == 1).mean())
+        result["roofline_encode"] = {
+            "kernel": "encode_kernel",
+            "hbm": {"achieved": bytes_enc / enc_mean / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": bytes_enc / enc_mean / hbm_peak, "bytes_per_launch": bytes_enc},
+            "alu": {"achieved": ops_enc / enc_mean / 1e12, "peak": alu_peak / 1e12, "unit": "Tops/s",
+                    "frac": ops_enc / enc_mean / alu_peak, "ops_per_launch": ops_enc},
+            "traffic": profile_traffic("encode_kernel"),
+        }
+    if e2e is not None:
+        result["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+    print(json.dumps(result), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def store_has_wide(wl) -> bool:
+    return bool((((wl.n_bits.astype(np.int64) + 1 + 31) // 32) > 9).any())
+
+
+def store_has_narrow(wl) -> bool:
+    return bool((((wl.n_bits.astype(np.int64) + 1 + 31) // 32) <= 9).any())
+
+
+def basis_bytes_touched(wl, store) -> int:
+    """Basis bytes of the distinct contexts the queries name, each read once."""
+    used = np.unique(wl.queries.ctx_id)
+    d = wl.n_bits.astype(np.int64)[used] + 1
+    wd = (d + 31) // 32
+    return int((d * (16 + 4 * wd) + 4 * wd).sum())
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_20532_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profile_traffic(kernel: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel sources (null otherwise)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------ CPU oracle
+
+def _sample(wl, target_rows: int, seed: int = 7):
+    rng = np.random.default_rng(seed)
+    perm = rng.permutation(wl.num_ctx)
+    acc = np.cumsum(wl.rows[perm])
+    k = int(np.searchsorted(acc, target_rows)) + 1
+    return np.sort(perm[:max(1, min(k, wl.num_ctx))])
+
+
+def _subset(wl, ctxs, qsel):
+    """Compact copy of the rows (and queries) of the sampled contexts."""
+    n = wl.n_bits[ctxs]
+    W = (n.astype(np.int64) + 31) // 32
+    batches, xs, ys = [], [], []
+    xbase = ybase = 0
+    for ro, xo in wl.batches:
+        cnt = ro[ctxs + 1] - ro[ctxs]
+        r_off = np.zeros(len(ctxs) + 1, np.int64)
+        r_off[1:] = ybase + np.cumsum(cnt)
+        r_off[0] = ybase
+        x_off = xbase + np.concatenate([[0], np.cumsum(cnt * W)[:-1]])
+        yi = np.concatenate([np.arange(ro[c], ro[c + 1]) for c in ctxs])
+        xi = np.concatenate([np.arange(xo[c], xo[c] + k * w) for c, k, w in zip(ctxs, cnt, W)])
+        ys.append(wl.y[yi])
+        xs.append(wl.x[xi])
+        batches.append((r_off, x_off))
+        ybase += len(yi)
+        xbase += len(xi)
+    x = np.concatenate(xs)
+    y = np.concatenate(ys)
+    q = None
+    if qsel is not None and len(qsel):
+        remap = np.full(wl.num_ctx, -1, np.int32)
+        remap[ctxs] = np.arange(len(ctxs), dtype=np.int32)
+        q = (remap[wl.queries.ctx_id[qsel]], np.ascontiguousarray(wl.queries.x[qsel]))
+    return n, batches, x, y, q
+
+
+def _oracle_step(sub, threads):
+    """One oracle step on a prepared subset: learn, solve, encode (timed)."""
+    import oracle
+
+    n, batches, x, y, q = sub
+    t0 = time.perf_counter()
+    O = oracle.Oracle(n, threads=threads)
+    for ro, xo in batches:
+        O.learn(ro, xo, x, y)
+    O.solve()
+    if q is not None:
+        O.encode(q[0], q[1])
+    t = time.perf_counter() - t0
+    O.close()
+    return t
+
+
+def _queries_for(wl, ctxs, frac):
+    if wl.queries is None:
+        return None
+    ins = np.flatnonzero(np.isin(wl.queries.ctx_id, ctxs))
+    return ins[: int(len(wl.queries.ctx_id) * frac)]
+
+
+def cpu_baseline(wl, seconds: float) -> dict:
+    """The oracle as it stands, on the host cores, on a bounded sample."""
+    threads = os.cpu_count() or 1
+    probe = _sample(wl, 300_000, seed=1)
+    t = _oracle_step(_subset(wl, probe, None), threads)
+    rate = wl.rows[probe].sum() / max(t, 1e-6)
+    target = int(min(wl.total_rows, max(100_000, rate * seconds)))
+    ctxs = _sample(wl, target, seed=2)
+    frac = wl.rows[ctxs].sum() / wl.total_rows
+    qsel = _queries_for(wl, ctxs, frac)
+    t = _oracle_step(_subset(wl, ctxs, qsel), threads)
+    rows = int(wl.rows[ctxs].sum())
+    return {"value": rows / t, "unit": "rows/s", "cores": threads, "kind": "oracle",
+            "sample": f"{len(ctxs)} of {wl.num_ctx} contexts ({rows} rows, {0 if qsel is None else len(qsel)} "
+                      f"queries, {100 * frac:.1f}% of the step), learn + solve + encode, {t:.1f} s"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+
+    oracle.build()
+    wl = workload_for(args.config, 0)
+    threads = os.cpu_count() or 1
+    ctxs = _sample(wl, args.ref_rows, seed=3)
+    frac = wl.rows[ctxs].sum() / wl.total_rows
+    qsel = _queries_for(wl, ctxs, frac)
+    sub = _subset(wl, ctxs, qsel)
+    for _ in range(args.warmup):
+        _oracle_step(sub, threads)
+    times = [_oracle_step(sub, threads) for _ in range(args.steps)]
+    rows = int(wl.rows[ctxs].sum())
+    ms = 1e3 * statistics.mean(times)
+    value = rows / (ms / 1e3)
+    sample = (f"{len(ctxs)} of {wl.num_ctx} contexts ({rows} rows, {0 if qsel is None else len(qsel)} queries, "
+              f"{100 * frac:.1f}% of the step) per step")
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded planted affine maps)",
+           "config": describe(args.config, wl),
+           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": threads, "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, choices=[1, 2, 3, 5], default=3)
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-rows", type=int, default=4_000_000)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-probe", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

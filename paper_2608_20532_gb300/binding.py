@@ -35,7 +35,7 @@ F2_OPT_WARP_BASIS_BYTES = 2
 EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
-    "f2_store_export", "f2_store_import", "f2_set_option",
+    "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3",
 )
 
 _lib = None
@@ -77,6 +77,7 @@ def load_library(path: Optional[str] = None):
         "f2_store_export": ([P, P, ctypes.POINTER(ctypes.c_size_t), P], ctypes.c_int),
         "f2_store_import": ([P, P, ctypes.c_size_t, P], ctypes.c_int),
         "f2_set_option": ([P, ctypes.c_int, i64], ctypes.c_int),
+        "f2_peak_lop3": ([P, i32, i32, ctypes.POINTER(i64), P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -216,6 +217,14 @@ class Store:
     def import_state(self, data: bytes, stream=None):
         buf = ctypes.create_string_buffer(data, len(data))
         _check(self._lib.f2_store_import(self._h, buf, len(data), _stream(stream)), "f2_store_import")
+
+
+def peak_lop3(blocks: int, iters: int, out: torch.Tensor, stream=None) -> int:
+    """Launch the integer-pipe probe; returns the LOP3 lane-operations it executes."""
+    n = ctypes.c_int64(0)
+    _check(load_library().f2_peak_lop3(_dptr(out), int(blocks), int(iters), ctypes.byref(n), _stream(stream)),
+           "f2_peak_lop3")
+    return int(n.value)
 
 
 def to_device(a: np.ndarray, device) -> torch.Tensor:

@@ -11,10 +11,14 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def _declared():
-    with open(os.path.join(ROOT, "include", "f2gpu.h")) as f:
-        text = f.read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(f2_[a-z_]+)\s*\(", text)))
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for h in sorted(os.listdir(inc)):
+        if h.endswith(".h"):
+            with open(os.path.join(inc, h)) as f:
+                text = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
+            names |= set(re.findall(r"\b(f2_[a-z0-9_]+)\s*\(", text))
+    return sorted(names)
 
 
 @pytest.fixture(scope="module")
@@ -39,7 +43,7 @@ def test_library_exports_every_declared_symbol(libpath):
     for name in _declared():
         assert hasattr(lib, name), name
     out = subprocess.run(["nm", "-D", "--defined-only", libpath], capture_output=True, text=True).stdout
-    exported = set(re.findall(r"\bT (f2_[a-z_]+)", out))
+    exported = set(re.findall(r"\bT (f2_[a-z0-9_]+)", out))
     assert set(_declared()) <= exported
 
 
