@@ -195,6 +195,55 @@ enum f2_option {
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 
+/*
+ * Allocation-free learning (the paper has no counterpart; this is a
+ * deployment aid).  Some callers cannot call cudaMalloc: processes whose
+ * device memory is entirely pre-reserved by a pooling allocator (a
+ * framework's caching allocator, an inference server's arena), where an
+ * extra cudaMalloc fails or breaks the memory budget, and latency-critical
+ * code that must not pay the implicit device synchronization that
+ * cudaMalloc and cudaFree can cause.  f2_learn_batched_noalloc performs one
+ * call of f2_learn_batched without any allocation: no store, no cudaMalloc,
+ * cudaFree or allocating library routine.  The caller owns every buffer;
+ * the scheduling scratch (context descriptors, work queues, counters) lives
+ * in one fixed, file-scope device array of the library, sized for
+ * F2_NOALLOC_MAX_CTX contexts (about 0.9 MB), that every GPU which loads the
+ * library holds until the process exits.
+ *
+ *   num_ctx        in [0, F2_NOALLOC_MAX_CTX]; larger values are rejected
+ *                  with F2_ERR_INVALID_ARG before anything is enqueued.
+ *   n_bits_host    host int32[num_ctx], each in [1, 1024] (F2_ERR_NBITS).
+ *   flags          0 or F2_FLAG_RAW_FEATURES, as for f2_create.
+ *   state (device, caller-owned, in/out, canonical layout of f2_get_basis;
+ *          sizes from d_c = n_c + 1 (n_c for raw rows), Wd_c = ceil(d_c/32)):
+ *     rank_dev int32[num_ctx], pivot_mask_dev uint32[sum Wd_c],
+ *     basis_x_dev uint32[sum d_c*Wd_c], basis_z_dev uint32[4*sum d_c]
+ *     (16-byte aligned), contra_dev uint8[num_ctx], first_contra_dev
+ *     int64[num_ctx], n_contra_dev uint64[num_ctx], rows_seen_dev
+ *     int64[num_ctx].  Before the first call every array must be zero except
+ *     first_contra_dev, which must be -1 everywhere; each call then continues
+ *     the streams exactly as f2_learn_batched continues a store's.
+ *   status_dev     device int32: set to F2_OK by the call, then receives the
+ *                  first device-detected error (F2_ERR_ROWS).
+ *   row_off_dev, x_dev, x_off_dev, y_dev, total_rows, total_x_words: one
+ *                  CSR batch, exactly as for f2_learn_batched.
+ * The first call on a device (per process) looks up the device address of
+ * the scratch array with cudaGetSymbolAddress; make that first call before
+ * any stream capture.  Every call shares the one scratch array and
+ * rewrites what it uses, so calls that overlap on the GPU (different
+ * streams, or different host threads) race: serialize them.  Results are
+ * bit-identical to f2_learn_batched on the same inputs.
+ * Errors: F2_ERR_INVALID_ARG, F2_ERR_NBITS, F2_ERR_ALIGN, F2_ERR_CUDA.
+ */
+#define F2_NOALLOC_MAX_CTX 16384
+int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
+                             int32_t* rank_dev, uint32_t* pivot_mask_dev, uint32_t* basis_x_dev,
+                             uint32_t* basis_z_dev, uint8_t* contra_dev, int64_t* first_contra_dev,
+                             uint64_t* n_contra_dev, int64_t* rows_seen_dev, int32_t* status_dev,
+                             const int64_t* row_off_dev, const uint32_t* x_dev, const int64_t* x_off_dev,
+                             const uint32_t* y_dev, int64_t total_rows, int64_t total_x_words,
+                             f2_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

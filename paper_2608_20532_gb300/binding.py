@@ -35,7 +35,7 @@ F2_OPT_WARP_BASIS_BYTES = 2
 EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
-    "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3",
+    "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3", "f2_learn_batched_noalloc",
 )
 
 _lib = None
@@ -78,6 +78,7 @@ def load_library(path: Optional[str] = None):
         "f2_store_import": ([P, P, ctypes.c_size_t, P], ctypes.c_int),
         "f2_set_option": ([P, ctypes.c_int, i64], ctypes.c_int),
         "f2_peak_lop3": ([P, i32, i32, ctypes.POINTER(i64), P], ctypes.c_int),
+        "f2_learn_batched_noalloc": ([i32, P, u32] + [P] * 9 + [P, P, P, P, i64, i64, P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)

@@ -664,3 +664,237 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     return F2_OK;
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of f2_learn_batched (no counterpart in the paper;
+// see f2_learn_batched_noalloc in f2gpu.h).  The scheduling scratch that a
+// store would own lives in one file-scope device array of fixed capacity.
+
+#include <mutex>
+
+namespace {
+
+struct NoallocScratch {
+    CtxDesc desc[F2_NOALLOC_MAX_CTX];
+    int32_t n_bits[F2_NOALLOC_MAX_CTX];
+    int32_t queue[F2_NOALLOC_MAX_CTX];
+    int32_t keybuf[F2_NOALLOC_MAX_CTX];
+    int counters[16];
+};
+
+// Device storage for the scratch; in host code this name is only a symbol
+// handle, its device address comes from cudaGetSymbolAddress.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[sizeof(NoallocScratch)];
+
+constexpr int NOALLOC_MAX_DEVICES = 64;
+constexpr int NOALLOC_NARROW_SMEM_DEFAULT = 4 * LEARN_WARPS * (8192 / 4);
+constexpr int NOALLOC_HEAVY_ROWS = 4096;
+constexpr int NOALLOC_WARP_REGION_WORDS = 8192 / 4;
+
+struct NoallocDevice {
+    NoallocScratch* scratch;
+    int num_sms;
+    bool ready;
+};
+NoallocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
+std::mutex g_noalloc_mu;
+
+// Once per device (with that device current): resolve the scratch address.
+int noalloc_setup(NoallocDevice** out)
+{
+    int device = -1;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    if (device < 0 || device >= NOALLOC_MAX_DEVICES) return F2_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoallocDevice& d = g_noalloc_dev[device];
+    if (!d.ready) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || p == nullptr) return e != cudaSuccess ? f2_cuda_status(e) : F2_ERR_CUDA;
+        int sms = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        d.scratch = static_cast<NoallocScratch*>(p);
+        d.num_sms = sms;
+        d.ready = true;
+    }
+    *out = &d;
+    return F2_OK;
+}
+
+// Context descriptors and canonical offsets (exclusive prefix sums of d,
+// d*wd and wd) for up to F2_NOALLOC_MAX_CTX contexts, one block.
+__global__ void __launch_bounds__(1024) noalloc_desc_kernel(const int32_t* __restrict__ n_bits, int C, uint32_t raw,
+                                                            CtxDesc* __restrict__ desc)
+{
+    constexpr int PER = (F2_NOALLOC_MAX_CTX + 1023) / 1024;
+    __shared__ long long wsum[3][32];
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    long long a = 0, b = 0, c = 0;
+    for (int i = 0; i < PER; ++i) {
+        const int k = t * PER + i;
+        if (k < C) {
+            const int n = n_bits[k];
+            const int d = raw ? n : n + 1;
+            const int wd = (d + 31) / 32;
+            a += d;
+            b += (long long)d * wd;
+            c += wd;
+        }
+    }
+    long long ia = a, ib = b, ic = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long va = __shfl_up_sync(FULL, ia, o), vb = __shfl_up_sync(FULL, ib, o),
+                        vc = __shfl_up_sync(FULL, ic, o);
+        if (lane >= o) {
+            ia += va;
+            ib += vb;
+            ic += vc;
+        }
+    }
+    if (lane == 31) {
+        wsum[0][warp] = ia;
+        wsum[1][warp] = ib;
+        wsum[2][warp] = ic;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        long long sa = wsum[0][lane], sb = wsum[1][lane], sc = wsum[2][lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long va = __shfl_up_sync(FULL, sa, o), vb = __shfl_up_sync(FULL, sb, o),
+                            vc = __shfl_up_sync(FULL, sc, o);
+            if (lane >= o) {
+                sa += va;
+                sb += vb;
+                sc += vc;
+            }
+        }
+        wsum[0][lane] = sa - wsum[0][lane];
+        wsum[1][lane] = sb - wsum[1][lane];
+        wsum[2][lane] = sc - wsum[2][lane];
+    }
+    __syncthreads();
+    long long ea = wsum[0][warp] + ia - a, eb = wsum[1][warp] + ib - b, ec = wsum[2][warp] + ic - c;
+    for (int i = 0; i < PER; ++i) {
+        const int k = t * PER + i;
+        if (k < C) {
+            CtxDesc cd;
+            cd.n = n_bits[k];
+            cd.d = raw ? cd.n : cd.n + 1;
+            cd.wd = (cd.d + 31) / 32;
+            cd.xw = (cd.n + 31) / 32;
+            cd.slot_off = ea;
+            cd.xw_off = eb;
+            cd.pw_off = ec;
+            cd.pad = 0;
+            desc[k] = cd;
+            ea += cd.d;
+            eb += (long long)cd.d * cd.wd;
+            ec += cd.wd;
+        }
+    }
+}
+
+}  // namespace
+
+extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
+                                        int32_t* rank_dev, uint32_t* pivot_mask_dev, uint32_t* basis_x_dev,
+                                        uint32_t* basis_z_dev, uint8_t* contra_dev, int64_t* first_contra_dev,
+                                        uint64_t* n_contra_dev, int64_t* rows_seen_dev, int32_t* status_dev,
+                                        const int64_t* row_off_dev, const uint32_t* x_dev, const int64_t* x_off_dev,
+                                        const uint32_t* y_dev, int64_t total_rows, int64_t total_x_words,
+                                        f2_stream_t stream)
+{
+    if (num_ctx < 0 || num_ctx > F2_NOALLOC_MAX_CTX || (flags & ~F2_FLAG_RAW_FEATURES) || total_rows < 0 ||
+        total_x_words < 0 || !status_dev)
+        return F2_ERR_INVALID_ARG;
+    if (num_ctx == 0) return F2_OK;
+    if (!n_bits_host || !rank_dev || !pivot_mask_dev || !basis_x_dev || !basis_z_dev || !contra_dev ||
+        !first_contra_dev || !n_contra_dev || !rows_seen_dev || !row_off_dev || !x_off_dev ||
+        (!x_dev && total_x_words) || (!y_dev && total_rows))
+        return F2_ERR_INVALID_ARG;
+    if (!is_aligned(row_off_dev, 8) || !is_aligned(x_off_dev, 8) || !is_aligned(x_dev, 4) || !is_aligned(y_dev, 16) ||
+        !is_aligned(basis_z_dev, 16) || !is_aligned(first_contra_dev, 8) || !is_aligned(n_contra_dev, 8) ||
+        !is_aligned(rows_seen_dev, 8) || !is_aligned(rank_dev, 4) || !is_aligned(pivot_mask_dev, 4) ||
+        !is_aligned(basis_x_dev, 4) || !is_aligned(status_dev, 4))
+        return F2_ERR_ALIGN;
+    const bool raw = (flags & F2_FLAG_RAW_FEATURES) != 0;
+    int max_narrow_bytes = 0, max_d = 0, n_wide = 0, n_narrow = 0;
+    for (int32_t c = 0; c < num_ctx; ++c) {
+        const int n = n_bits_host[c];
+        if (n < 1 || n > MAX_N) return F2_ERR_NBITS;
+        const int d = raw ? n : n + 1;
+        const int wd = (d + 31) / 32;
+        if (d > max_d) max_d = d;
+        if (wd > NARROW_WD) {
+            ++n_wide;
+        } else {
+            ++n_narrow;
+            const int bytes = 4 * (CTL_WORDS + d * row_stride(wd));
+            if (bytes > max_narrow_bytes) max_narrow_bytes = bytes;
+        }
+    }
+    NoallocDevice* nd = nullptr;
+    int rc = noalloc_setup(&nd);
+    if (rc != F2_OK) return rc;
+    NoallocScratch* sc = nd->scratch;
+    cudaStream_t cs = (cudaStream_t)stream;
+
+    cudaError_t e = cudaMemsetAsync(status_dev, 0, sizeof(int32_t), cs);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(sc->n_bits, n_bits_host, sizeof(int32_t) * (size_t)num_ctx, cudaMemcpyHostToDevice, cs);
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    noalloc_desc_kernel<<<1, 1024, 0, cs>>>(sc->n_bits, num_ctx, raw ? 1u : 0u, sc->desc);
+
+    StoreDev sd;
+    sd.desc = sc->desc;
+    sd.rank = rank_dev;
+    sd.contra = contra_dev;
+    sd.first_contra = reinterpret_cast<long long*>(first_contra_dev);
+    sd.n_contra = reinterpret_cast<unsigned long long*>(n_contra_dev);
+    sd.rows_seen = reinterpret_cast<long long*>(rows_seen_dev);
+    sd.pivot = pivot_mask_dev;
+    sd.bx = basis_x_dev;
+    sd.bz = reinterpret_cast<uint4*>(basis_z_dev);
+    sd.status = status_dev;
+    sd.num_ctx = num_ctx;
+    sd.raw = raw ? 1u : 0u;
+    plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off_dev, x_off_dev, total_rows, total_x_words, NOALLOC_WARP_REGION_WORDS,
+                                    NOALLOC_HEAVY_ROWS, sc->queue, sc->keybuf, sc->counters);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return f2_cuda_status(e);
+
+    LearnArgs la;
+    la.row_off = row_off_dev;
+    la.x_off = x_off_dev;
+    la.x = x_dev;
+    la.y = reinterpret_cast<const uint4*>(y_dev);
+    la.queue = sc->queue;
+    la.counters = sc->counters;
+    la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
+    if (n_narrow) {
+        const int smem = max_narrow_bytes > NOALLOC_NARROW_SMEM_DEFAULT ? max_narrow_bytes : NOALLOC_NARROW_SMEM_DEFAULT;
+        e = cudaFuncSetAttribute(learn_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        int per_sm = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, learn_narrow_kernel, LEARN_WARPS * 32, smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        if (per_sm < 1) per_sm = 1;
+        learn_narrow_kernel<<<nd->num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    if (n_wide) {
+        const int smem = 4 * (CTL_WORDS + max_d * row_stride(WIDE_WD));
+        e = cudaFuncSetAttribute(learn_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        const int blocks = n_wide < nd->num_sms ? n_wide : nd->num_sms;
+        learn_wide_kernel<<<blocks, WIDE_WARPS * 32, smem, cs>>>(sd, la);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    return F2_OK;
+}
