@@ -122,7 +122,10 @@ int f2_sizes(const f2_store* store, int32_t* num_ctx, int64_t* slots, int64_t* b
  * index of the first contradicting row (counted over the context's whole
  * stream, across calls, from 0) and the number of contradicting rows.
  * Contradicting rows are not inserted; learning continues after them.
- * Scratch: the scheduling queue allocated by f2_create (one call at a time).
+ * At most 2^31 - 1 rows per context per call (larger contexts: F2_ERR_ROWS).
+ * Scratch: the scheduling queues allocated by f2_create and 8 bytes per row
+ * of y_dev (grown stream-ordered with cudaMallocAsync when total_rows exceeds
+ * the previous capacity); calls on one store must not overlap.
  * Errors: F2_ERR_INVALID_ARG (NULL pointer or negative size), F2_ERR_ALIGN
  * (y_dev not 16-byte aligned, offsets not 8-byte aligned), F2_ERR_CUDA.
  */
@@ -191,7 +194,10 @@ int f2_store_import(f2_store* store, const void* host_buf, size_t size, f2_strea
 /* Scheduling knobs of f2_learn_batched (performance only, never results). */
 enum f2_option {
     F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA */
-    F2_OPT_WARP_BASIS_BYTES = 2 /* largest basis (bytes of shared memory) handled by one warp */
+    F2_OPT_WARP_BASIS_BYTES = 2, /* shared memory (bytes) of one warp-owned context */
+    F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context */
+    F2_OPT_DEDUP = 4             /* 1 (default): eliminate only the first occurrence of each distinct
+                                    row and classify its repeats with it; 0: eliminate every row */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

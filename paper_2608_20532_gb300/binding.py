@@ -30,6 +30,8 @@ F2_ERR_STRIDE = 9
 F2_FLAG_RAW_FEATURES = 1
 F2_OPT_HEAVY_ROWS = 1
 F2_OPT_WARP_BASIS_BYTES = 2
+F2_OPT_WARP_WORK = 3
+F2_OPT_DEDUP = 4
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

@@ -17,17 +17,20 @@ constexpr int NARROW_WD = 9;         // widest row (32-bit words) handled by the
 constexpr int LEARN_WARPS = 8;       // warps per CTA of the narrow learn kernel
 constexpr int WIDE_WARPS = 8;        // warps per CTA of the wide learn kernel
 constexpr int PLAN_BUCKETS = 48;     // log2(work) buckets for longest-first ordering
+constexpr int DEFAULT_WARP_REGION_BYTES = 12288;  // shared memory of one warp-owned context
+constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA
+constexpr long long DEFAULT_WARP_WORK = 131072;   // largest rows x d handled by one warp
 
 // Scheduling counters written by the plan kernel, read by the learn kernels.
 enum Counter {
-    CNT_HEAD_CTA = 0,  // next item of the CTA queue (narrow contexts, one CTA each)
-    CNT_HEAD_WIDE = 1, // next item of the wide queue
-    CNT_HEAD_WARP = 2, // next item of the warp queue
-    CNT_BEGIN = 3,     // 3 + class: first queue slot of each class
-    CNT_COUNT = 6,     // 6 + class: number of contexts of each class
-    CNT_TOTAL = 9
+    CNT_HEAD = 0,   // + class: next queue item of each class
+    CNT_BEGIN = 8,  // + class: first queue slot of each class
+    CNT_COUNT = 16, // + class: number of contexts of each class
+    CNT_WORDS = 32
 };
-enum Class { CLS_CTA = 0, CLS_WIDE = 1, CLS_WARP = 2 };
+// Work classes: elimination by a CTA / the wide kernel / a warp, and dedup
+// by a CTA / a warp.
+enum Class { CLS_CTA = 0, CLS_WIDE = 1, CLS_WARP = 2, CLS_DD_CTA = 3, CLS_DD_WARP = 4, NUM_CLASSES = 5 };
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {
@@ -81,6 +84,8 @@ struct f2_store {
     int64_t pivot_words;
     int64_t heavy_rows;
     int64_t warp_basis_bytes;
+    int64_t warp_work;
+    int dedup;              // run the duplicate pass before elimination
     std::vector<int32_t> n_bits;
     std::vector<int64_t> slot_off, xw_off, pw_off;
     // device memory
@@ -98,6 +103,10 @@ struct f2_store {
     int32_t* queue;
     int32_t* keybuf;
     int* counters;
+    int32_t* rep_count;     // representatives per context (pass 1 output)
+    int32_t* rep_list;      // per-row scratch of pass 1 (capacity rep_capacity rows)
+    int32_t* rep_dup;
+    int64_t rep_capacity;
 
     f2::StoreDev dev() const
     {

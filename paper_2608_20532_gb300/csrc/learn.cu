@@ -1,35 +1,43 @@
 // Batched streaming Gaussian elimination over GF(2) (Sec. 2.2) on sm_103a.
 //
-// Every context owns a reduced basis B[k] = (r_k, z_k), kept in shared memory
-// while its rows stream in.  A group of lanes processes the rows of one
-// context in rounds of 32 rows per warp:
+// A call runs two passes over each context's rows (stream order = CSR order):
 //
-//  1. reduce: each lane reduces its row against the basis as it stood at the
-//     start of the round (the snapshot).  The basis is reduced (RREF, the
-//     paper's step (5)), so the rows to XOR are exactly the pivots set in the
-//     row itself; the warp walks the union of those pivots and every lane
-//     XORs the broadcast row under its own bit (shared-memory broadcast, no
-//     bank conflicts);
-//  2. classify: a zero feature residual means the row lies in the span of
-//     the snapshot.  The map T fixed by the snapshot never changes afterwards
-//     (rows that contradict it are not inserted, insertions only extend it),
-//     so such a row is classified exactly as the one-row-at-a-time algorithm
-//     would classify it: zero word residual -> redundant, else contradiction
-//     (Sec. 2.2 steps (2)-(3));
-//  3. insert: the remaining rows (candidates) are eliminated among themselves
-//     in stream order inside the warp (lane order), which reproduces step (4)
-//     for each of them, then merged: the new rows are stored at their pivot
-//     slots and every older row is cleared at the new pivot columns (step
-//     (5)).  The result is the same reduced basis, with the same z_k, as the
-//     sequential algorithm's.
+//  Pass 1 (dedup): the first occurrence of every distinct observation (x, y)
+//  of a context is its representative; later equal rows are its duplicates.
+//  A duplicate needs no elimination: its row equals an earlier row, so it
+//  lies in the span when it arrives and is classified exactly as that earlier
+//  row was -- redundant if the representative was consistent, a
+//  contradiction if the representative was one (T never changes on the span).
+//  Equality is decided by comparing the full rows (hash tables in shared
+//  memory only propose the candidates), so the pass is exact.
 //
-// Contexts with few rows and a small basis get one warp each (many per CTA);
-// heavy contexts get a whole CTA whose warps reduce 256 rows per round and
-// insert their candidates warp by warp in stream order.  Contexts wider than
-// 288 bits (d up to 1025) run in a separate wide kernel, one CTA each.  A
-// single-block plan kernel validates the CSR batch and orders contexts
-// longest-first into one queue per class.
+//  Pass 2 (elimination) streams the representatives of each context, in
+//  order, through a reduced basis B[k] = (r_k, z_k) held in shared memory:
+//   1. reduce: each lane reduces its row against the basis as it stood at
+//      the start of the round (the snapshot).  The basis is reduced (RREF,
+//      the paper's step (5)), so the rows to XOR are exactly the pivots set
+//      in the row itself; the warp walks the union of those pivots and every
+//      lane XORs the broadcast row under its own bit;
+//   2. classify: a zero feature residual means the row lies in the span of
+//      the snapshot, and the map T fixed by the snapshot never changes
+//      afterwards (contradicting rows are not inserted, insertions only
+//      extend it), so the classification equals the one-row-at-a-time one:
+//      zero word residual -> redundant, else contradiction (steps (2)-(3)).
+//      A contradicting representative counts once for itself and once per
+//      duplicate; its index is the first of them;
+//   3. insert: the remaining rows (candidates) are eliminated among
+//      themselves in stream order inside the warp (step (4)), then merged:
+//      new rows go to their pivot slots and every older row is cleared at
+//      the new pivot columns (step (5)).  The basis, including every z_k, is
+//      the sequential algorithm's.
+//
+// Both passes give one warp to small contexts (many per CTA) and a whole CTA
+// to large ones; contexts wider than 288 bits (d up to 1025) are eliminated
+// by a separate wide kernel.  Single-block plan kernels validate the CSR
+// batch and order the work longest-first.
 #include <limits.h>
+
+#include <mutex>
 
 #include "f2_internal.cuh"
 
@@ -42,20 +50,51 @@ struct LearnArgs {
     const int64_t* x_off;
     const uint32_t* x;
     const uint4* y;
+    const int32_t* rep_list;   // representatives (row indices, per-context at row_off[c]); NULL = every row
+    const int32_t* rep_dup;    // duplicates of each representative (NULL = none)
+    const int32_t* rep_count;  // representatives per context (NULL = all rows)
     const int32_t* queue;
     int* counters;
     int warp_region_words;
 };
 
-// Shared-memory control area of a CTA-mode context (32-bit words).
+struct DedupArgs {
+    const int64_t* row_off;
+    const int64_t* x_off;
+    const uint32_t* x;
+    const uint4* y;
+    int32_t* rep_list;
+    int32_t* rep_dup;
+    int32_t* rep_count;
+    const int32_t* queue;
+    int* counters;
+};
+
+// Shared-memory control area of an elimination group (32-bit words).
 constexpr int CTL_P = 0;       // pivot mask, 48 words
 constexpr int CTL_NPR = 48;    // pivots added during the current round, 48 words
-constexpr int CTL_CAND = 96;   // candidate ballots, 2 x 32 words (round parity)
+constexpr int CTL_CAND = 96;   // per-warp candidate ballots, 32 words
 constexpr int CTL_RANK = 160;  // rank
 constexpr int CTL_CNT = 162;   // contradiction count (uint64, 8-byte aligned)
 constexpr int CTL_FIRST = 164; // first contradiction index (int64)
 constexpr int CTL_WORDS = 176; // size of the control area (16-byte multiple)
-constexpr int WARP_CTL = 16;   // control words in front of a warp-mode basis
+
+// Pass 1: 16 warps per CTA, one CTA per SM.  A warp-owned context (at most
+// DD_WARP_MAX_ROWS rows) gets a table of next_pow2(2T) entries in a 12 KB
+// region; a CTA-owned context a table of up to DD_CTA_E entries.  Entry =
+// (fingerprint, row index) plus a duplicate counter: 12 bytes.
+constexpr int DD_THREADS = 512;
+constexpr int DD_WARPS = DD_THREADS / 32;
+constexpr int DD_WARP_MAX_ROWS = 512;
+constexpr int DD_WARP_E = 1024;
+constexpr int DD_WARP_REGION = 3 * DD_WARP_E;   // words
+constexpr int DD_CTA_E = 16384;
+constexpr int DD_SMEM = 4 * 3 * DD_CTA_E;       // bytes (also 16 warp regions)
+constexpr int DD_K = 4;                         // rows per thread in flight
+constexpr int DEDUP_PROBES = 8;                 // linear-probe limit
+static_assert(DD_WARPS * DD_WARP_REGION * 4 <= DD_SMEM, "warp regions exceed the dedup shared memory");
+
+__host__ __device__ __forceinline__ int elim_words(int d, int wd) { return CTL_WORDS + d * row_stride(wd); }
 
 __device__ __forceinline__ bool nonzero4(const uint4& v) { return (v.x | v.y | v.z | v.w) != 0u; }
 
@@ -83,14 +122,11 @@ __device__ __forceinline__ uint64_t mixed_words(const uint32_t (&P)[WD], int d, 
     return m;
 }
 
-// Load row i of a context into (q, y): q = [1 || x] (index 0 = constant),
-// or x itself for raw feature rows.  Lanes past the end load zeros.
+// Feature words exactly as supplied (bits >= n cleared), and the word.
 template <int WD>
-__device__ __forceinline__ void load_row(const uint32_t* __restrict__ xrow, const uint4* __restrict__ yrow,
-                                         bool valid, int n, int xw, uint32_t raw, uint32_t (&q)[WD],
-                                         uint4& y)
+__device__ __forceinline__ void load_raw(const uint32_t* __restrict__ xrow, const uint4* __restrict__ yrow,
+                                         bool valid, int n, int xw, uint32_t (&xin)[WD], uint4& y)
 {
-    uint32_t xin[WD];
 #pragma unroll
     for (int v = 0; v < WD; ++v) {
         uint32_t t = 0;
@@ -98,6 +134,13 @@ __device__ __forceinline__ void load_row(const uint32_t* __restrict__ xrow, cons
         if (v == xw - 1 && (n & 31)) t &= (1u << (n & 31)) - 1u;
         xin[v] = t;
     }
+    y = valid ? __ldg(yrow) : make_uint4(0, 0, 0, 0);
+}
+
+// q = [1 || x] (index 0 = constant) or x itself for raw feature rows.
+template <int WD>
+__device__ __forceinline__ void make_q(const uint32_t (&xin)[WD], bool valid, uint32_t raw, uint32_t (&q)[WD])
+{
     if (raw) {
 #pragma unroll
         for (int v = 0; v < WD; ++v) q[v] = xin[v];
@@ -106,7 +149,217 @@ __device__ __forceinline__ void load_row(const uint32_t* __restrict__ xrow, cons
 #pragma unroll
         for (int v = 1; v < WD; ++v) q[v] = (xin[v] << 1) | (xin[v - 1] >> 31);
     }
-    y = valid ? __ldg(yrow) : make_uint4(0, 0, 0, 0);
+}
+
+// 32-bit hash of an observation (feature words and word): FNV-1a over the
+// words, then a murmur-style finalizer.
+template <int WD>
+__device__ __forceinline__ uint32_t hash_row(const uint32_t (&xin)[WD], const uint4& y)
+{
+    uint32_t h = 0x811C9DC5u;
+#pragma unroll
+    for (int v = 0; v < WD; ++v) h = (h ^ xin[v]) * 0x01000193u;
+    h = (h ^ y.x) * 0x01000193u;
+    h = (h ^ y.y) * 0x01000193u;
+    h = (h ^ y.z) * 0x01000193u;
+    h = (h ^ y.w) * 0x01000193u;
+    h ^= h >> 16;
+    h *= 0x85EBCA6Bu;
+    h ^= h >> 13;
+    h *= 0xC2B2AE35u;
+    h ^= h >> 16;
+    return h;
+}
+
+template <bool CTA>
+__device__ __forceinline__ void group_sync()
+{
+    if (CTA) __syncthreads();
+    else __syncwarp();
+}
+
+// ------------------------------------------------------------------ pass 1
+
+__device__ __forceinline__ uint32_t fnv_step(uint32_t h, uint32_t w) { return (h ^ w) * 0x01000193u; }
+
+__device__ __forceinline__ uint32_t fmix32(uint32_t h)
+{
+    h ^= h >> 16;
+    h *= 0x85EBCA6Bu;
+    h ^= h >> 13;
+    h *= 0xC2B2AE35u;
+    h ^= h >> 16;
+    return h;
+}
+
+__device__ __forceinline__ uint32_t last_mask(int n) { return (n & 31) ? ((1u << (n & 31)) - 1u) : 0xffffffffu; }
+
+// Full comparison of rows i and j of a context (feature bits < n and word).
+__device__ __forceinline__ bool rows_equal(const uint32_t* __restrict__ xc, const uint4* __restrict__ yc, int xw, int n,
+                                           int64_t i, const uint4& yi, int64_t j)
+{
+    const uint4 yj = __ldg(yc + j);
+    if (yj.x != yi.x || yj.y != yi.y || yj.z != yi.z || yj.w != yi.w) return false;
+    const uint32_t lm = last_mask(n);
+    for (int v = 0; v < xw; ++v) {
+        const uint32_t m = (v == xw - 1) ? lm : 0xffffffffu;
+        if (((__ldg(xc + i * xw + v) ^ __ldg(xc + j * xw + v)) & m) != 0u) return false;
+    }
+    return true;
+}
+
+// Find the entry of row i's content, inserting it if absent.  Returns the
+// slot (whose index field ends as the smallest row index of that content), or
+// -1 when the probe limit is reached (the row then counts as its own
+// representative, which is always exact).
+__device__ __forceinline__ int dd_find_insert(uint2* tab, int E, uint32_t h, int64_t i, const uint4& yi,
+                                              const uint32_t* __restrict__ xc, const uint4* __restrict__ yc, int xw,
+                                              int n)
+{
+    const uint32_t fp = h | 1u;
+    uint32_t slot = (h >> 7) & (uint32_t)(E - 1);
+    for (int p = 0; p < DEDUP_PROBES; ++p, slot = (slot + 1) & (uint32_t)(E - 1)) {
+        uint2 e = tab[slot];
+        if (e.x == 0u) {
+            const unsigned long long want = ((unsigned long long)(uint32_t)i << 32) | fp;
+            const unsigned long long old = atomicCAS(reinterpret_cast<unsigned long long*>(tab + slot), 0ull, want);
+            if (old == 0ull) return (int)slot;
+            e.x = (uint32_t)old;
+            e.y = (uint32_t)(old >> 32);
+        }
+        if (e.x == fp && rows_equal(xc, yc, xw, n, i, yi, (int64_t)e.y)) {
+            if ((uint32_t)i < e.y) atomicMin(&tab[slot].y, (uint32_t)i);
+            return (int)slot;
+        }
+    }
+    return -1;
+}
+
+// One group (a warp, or the whole CTA) finds the representatives of context
+// c and writes them, in stream order, to rep_list[row_off[c] + k] with their
+// duplicate counts in rep_dup; rep_count[c] = number of representatives.
+template <bool CTA>
+__device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t* region, int E, int* wcnt)
+{
+    const int G = CTA ? (int)(blockDim.x >> 5) : 1;
+    const int lane = threadIdx.x & 31;
+    const int warp = CTA ? (int)(threadIdx.x >> 5) : 0;
+    const int t = 32 * warp + lane;
+    const int nt = 32 * G;
+    uint2* tab = reinterpret_cast<uint2*>(region);
+    int* D = reinterpret_cast<int*>(region + 2 * E);
+    const CtxDesc cd = s.desc[c];
+    const int xw = cd.xw, n = cd.n;
+    const int64_t r0 = a.row_off[c];
+    const int T = (int)(a.row_off[c + 1] - r0);
+    const uint32_t* xc = a.x + a.x_off[c];
+    const uint4* yc = a.y + r0;
+    const uint32_t lm = last_mask(n);
+    for (int e = t; e < E; e += nt) {
+        tab[e] = make_uint2(0u, 0u);
+        D[e] = 0;
+    }
+    group_sync<CTA>();
+    int nrep = 0;
+    for (int base = 0; base < T; base += nt * DD_K) {
+        int mine[DD_K];
+        uint32_t h[DD_K];
+        uint4 yv[DD_K];
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            const int i = base + j * nt + t;
+            h[j] = 0x811C9DC5u;
+            yv[j] = make_uint4(0, 0, 0, 0);
+            if (i < T) {
+                yv[j] = __ldg(yc + i);
+                for (int v = 0; v < xw; ++v)
+                    h[j] = fnv_step(h[j], __ldg(xc + (int64_t)i * xw + v) & ((v == xw - 1) ? lm : 0xffffffffu));
+                h[j] = fnv_step(fnv_step(fnv_step(fnv_step(h[j], yv[j].x), yv[j].y), yv[j].z), yv[j].w);
+                h[j] = fmix32(h[j]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            const int i = base + j * nt + t;
+            mine[j] = (i < T) ? dd_find_insert(tab, E, h[j], i, yv[j], xc, yc, xw, n) : -1;
+        }
+        group_sync<CTA>();
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            const int i = base + j * nt + t;
+            const bool valid = i < T;
+            const int rep = (valid && mine[j] >= 0) ? (int)tab[mine[j]].y : i;
+            const bool isrep = valid && rep == i;
+            if (valid && !isrep) atomicAdd(D + mine[j], 1);
+            const uint32_t bal = __ballot_sync(FULL, isrep);
+            int before = 0, total = __popc(bal);
+            if (CTA) {
+                if (lane == 0) wcnt[warp] = total;
+                __syncthreads();
+                total = 0;
+                for (int ww = 0; ww < G; ++ww) {
+                    const int v = wcnt[ww];
+                    if (ww < warp) before += v;
+                    total += v;
+                }
+                __syncthreads();
+            }
+            if (isrep) {
+                const int pos = nrep + before + __popc(bal & ((1u << lane) - 1u));
+                a.rep_list[r0 + pos] = i;
+                a.rep_dup[r0 + pos] = mine[j];
+            }
+            nrep += total;
+        }
+    }
+    group_sync<CTA>();
+    for (int k = t; k < nrep; k += nt) {
+        const int slot = a.rep_dup[r0 + k];
+        a.rep_dup[r0 + k] = (slot >= 0) ? D[slot] : 0;
+    }
+    if (t == 0) a.rep_count[c] = nrep;
+    group_sync<CTA>();
+}
+
+__device__ __forceinline__ int pow2_at_least(int v)
+{
+    int e = 64;
+    while (e < v) e <<= 1;
+    return e;
+}
+
+__global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupArgs a)
+{
+    extern __shared__ __align__(16) uint32_t smem[];
+    __shared__ int s_item;
+    __shared__ int wcnt[32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_cta = a.counters[CNT_COUNT + CLS_DD_CTA];
+    const int b_cta = a.counters[CNT_BEGIN + CLS_DD_CTA];
+    for (;;) {
+        __syncthreads();
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_CTA, 1);
+        __syncthreads();
+        const int item = s_item;
+        if (item >= n_cta) break;
+        const int c = a.queue[b_cta + item];
+        const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
+        int E = pow2_at_least(2 * T);
+        if (E > DD_CTA_E) E = DD_CTA_E;
+        dedup_ctx<true>(s, a, c, smem, E, wcnt);
+    }
+    const int n_w = a.counters[CNT_COUNT + CLS_DD_WARP];
+    const int b_w = a.counters[CNT_BEGIN + CLS_DD_WARP];
+    uint32_t* region = smem + warp * DD_WARP_REGION;
+    for (;;) {
+        int item = 0;
+        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_WARP, 1);
+        item = __shfl_sync(FULL, item, 0);
+        if (item >= n_w) break;
+        const int c = a.queue[b_w + item];
+        const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
+        dedup_ctx<false>(s, a, c, region, pow2_at_least(2 * T), nullptr);
+    }
 }
 
 // Step (1) against the snapshot S.  On return the residual is zero at every
@@ -174,7 +427,7 @@ __device__ __forceinline__ void reduce_new(uint32_t (&xr)[WD], uint4& yr, const 
 template <int WD>
 __device__ int insert_block(uint32_t (&xr)[WD], uint4& yr, uint32_t cand, uint32_t* __restrict__ S,
                             const uint32_t (&P)[WD], int d, int lane, long long idx, long long& first,
-                            unsigned long long& cnt, uint32_t (&NP)[WD])
+                            unsigned long long& cnt, uint32_t (&NP)[WD], bool& contra_lane, uint32_t weight)
 {
     constexpr int RS = row_stride(WD);
     int pk = -1;
@@ -189,8 +442,9 @@ __device__ int insert_block(uint32_t (&xr)[WD], uint4& yr, uint32_t cand, uint32
         const int k = __shfl_sync(FULL, mine, i);
         if (k < 0) {  // reduced to zero by rows inserted earlier in this block
             if (lane == i && nonzero4(yr)) {
-                ++cnt;
+                cnt += weight;
                 first = min(first, idx);
+                contra_lane = true;
             }
             continue;
         }
@@ -310,91 +564,52 @@ __device__ __forceinline__ void commit_stats(const StoreDev& s, int c, long long
     }
 }
 
-// One warp owns context c.
+// ------------------------------------------------------------------ pass 2
+
+// Context c's basis into shared memory (a context of rank 0 has an all-zero
+// stored basis, so it is cleared instead of read).
 template <int WD>
-__device__ void learn_ctx_warp(const StoreDev& s, const LearnArgs& a, int c, uint32_t* region, int lane)
+__device__ void basis_in(const StoreDev& s, const CtxDesc& cd, uint32_t* S, int t, int nt, bool empty)
 {
-    const CtxDesc cd = s.desc[c];
-    uint32_t* S = region + WARP_CTL;
-    basis_to_smem<WD>(s, cd, S, lane, 32);
-    uint32_t P[WD];
-#pragma unroll
-    for (int v = 0; v < WD; ++v) P[v] = (v < cd.wd) ? s.pivot[cd.pw_off + v] : 0u;
-    __syncwarp();
-    uint64_t mixed = mixed_words<WD>(P, cd.d, cd.wd);
-    int rank = s.rank[c];
-    const long long seen = s.rows_seen[c];
-    const int64_t r0 = a.row_off[c];
-    const int64_t T = a.row_off[c + 1] - r0;
-    const uint32_t* xc = a.x + a.x_off[c];
-    const uint4* yc = a.y + r0;
-    long long first = LLONG_MAX;
-    unsigned long long cnt = 0;
-    for (int64_t base = 0; base < T; base += 32) {
-        const int64_t i = base + lane;
-        const bool valid = i < T;
-        uint32_t xr[WD];
-        uint4 yr;
-        load_row<WD>(xc + (valid ? i : 0) * cd.xw, yc + (valid ? i : 0), valid, cd.n, cd.xw, s.raw, xr, yr);
-        reduce_snapshot<WD>(xr, yr, S, P, mixed);
-        uint32_t nz = 0;
-#pragma unroll
-        for (int v = 0; v < WD; ++v) {
-            xr[v] &= ~P[v];
-            nz |= xr[v];
-        }
-        if (valid && !nz && nonzero4(yr)) {
-            ++cnt;
-            first = min(first, seen + i);
-        }
-        const uint32_t cand = __ballot_sync(FULL, valid && nz != 0u);
-        if (cand) {
-            uint32_t NP[WD];
-            rank += insert_block<WD>(xr, yr, cand, S, P, cd.d, lane, seen + i, first, cnt, NP);
-#pragma unroll
-            for (int v = 0; v < WD; ++v) P[v] |= NP[v];
-            mixed = mixed_words<WD>(P, cd.d, cd.wd);
-        }
+    constexpr int RS = row_stride(WD);
+    if (empty) {
+        for (int w = t; w < cd.d * RS; w += nt) S[w] = 0u;
+        return;
     }
-    __syncwarp();
-#pragma unroll
-    for (int v = 0; v < WD; ++v)
-        if (lane == v && v < cd.wd) s.pivot[cd.pw_off + v] = P[v];
-    basis_from_smem<WD>(s, cd, S, lane, 32);
-    warp_stats(first, cnt);
-    if (lane == 0) {
-        s.rank[c] = rank;
-        s.rows_seen[c] = seen + T;
-        commit_stats(s, c, first, cnt);
-    }
-    __syncwarp();
+    basis_to_smem<WD>(s, cd, S, t, nt);
 }
 
-// All warps of the CTA own context c.
-template <int WD>
-__device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint32_t* smem)
+// One group (a warp, or the whole CTA) streams the representatives of
+// context c through its basis.
+template <int WD, bool CTA>
+__device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t* region)
 {
-    const int t = threadIdx.x, nt = blockDim.x;
-    const int warp = t >> 5, lane = t & 31, nwarps = nt >> 5;
+    const int G = CTA ? (int)(blockDim.x >> 5) : 1;
+    const int lane = threadIdx.x & 31;
+    const int warp = CTA ? (int)(threadIdx.x >> 5) : 0;
+    const int t = 32 * warp + lane;
+    const int nt = 32 * G;
     const CtxDesc cd = s.desc[c];
-    uint32_t* Ps = smem + CTL_P;
-    uint32_t* NPR = smem + CTL_NPR;
-    uint32_t* candw = smem + CTL_CAND;
-    int* rank_s = reinterpret_cast<int*>(smem + CTL_RANK);
-    unsigned long long* cnt_s = reinterpret_cast<unsigned long long*>(smem + CTL_CNT);
-    long long* first_s = reinterpret_cast<long long*>(smem + CTL_FIRST);
-    uint32_t* S = smem + CTL_WORDS;
-    basis_to_smem<WD>(s, cd, S, t, nt);
+    uint32_t* ctl = region;
+    uint32_t* Ps = ctl + CTL_P;
+    uint32_t* NPR = ctl + CTL_NPR;
+    uint32_t* wc = ctl + CTL_CAND;
+    int* rank_s = reinterpret_cast<int*>(ctl + CTL_RANK);
+    unsigned long long* cnt_s = reinterpret_cast<unsigned long long*>(ctl + CTL_CNT);
+    long long* first_s = reinterpret_cast<long long*>(ctl + CTL_FIRST);
+    uint32_t* S = region + CTL_WORDS;
+    const int rank0 = s.rank[c];
+    basis_in<WD>(s, cd, S, t, nt, rank0 == 0);
     if (t < 48) {
-        Ps[t] = (t < cd.wd) ? s.pivot[cd.pw_off + t] : 0u;
-        NPR[t] = 0;
+        Ps[t] = (t < cd.wd && rank0 != 0) ? s.pivot[cd.pw_off + t] : 0u;
+        NPR[t] = 0u;
     }
     if (t == 0) {
-        *rank_s = s.rank[c];
-        *cnt_s = 0;
+        *rank_s = rank0;
+        *cnt_s = 0ull;
         *first_s = LLONG_MAX;
     }
-    __syncthreads();
+    group_sync<CTA>();
     uint32_t P[WD];
 #pragma unroll
     for (int v = 0; v < WD; ++v) P[v] = Ps[v];
@@ -402,17 +617,33 @@ __device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint
     const long long seen = s.rows_seen[c];
     const int64_t r0 = a.row_off[c];
     const int64_t T = a.row_off[c + 1] - r0;
+    const int R = a.rep_count ? a.rep_count[c] : (int)T;
+    const int32_t* reps = a.rep_list ? a.rep_list + r0 : nullptr;
+    const int32_t* dups = a.rep_dup ? a.rep_dup + r0 : nullptr;
     const uint32_t* xc = a.x + a.x_off[c];
     const uint4* yc = a.y + r0;
     long long first = LLONG_MAX;
     unsigned long long cnt = 0;
-    int par = 0;
-    for (int64_t base = 0; base < T; base += 32 * nwarps, par ^= 1) {
-        const int64_t i = base + 32 * warp + lane;
-        const bool valid = i < T;
+    // prefetched round
+    int nk = t;
+    bool nvalid = nk < R;
+    int ni = nvalid ? (reps ? __ldg(reps + nk) : nk) : 0;
+    uint32_t nw = (nvalid && dups) ? (uint32_t)__ldg(dups + nk) : 0u;
+    uint32_t xn[WD];
+    uint4 yn;
+    load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
+    for (int base = 0; base < R; base += nt) {
+        const bool valid = nvalid;
+        const int i = ni;
+        const uint32_t weight = 1u + nw;
         uint32_t xr[WD];
-        uint4 yr;
-        load_row<WD>(xc + (valid ? i : 0) * cd.xw, yc + (valid ? i : 0), valid, cd.n, cd.xw, s.raw, xr, yr);
+        make_q<WD>(xn, valid, s.raw, xr);
+        uint4 yr = yn;
+        nk += nt;
+        nvalid = nk < R;
+        ni = nvalid ? (reps ? __ldg(reps + nk) : nk) : 0;
+        nw = (nvalid && dups) ? (uint32_t)__ldg(dups + nk) : 0u;
+        load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
         reduce_snapshot<WD>(xr, yr, S, P, mixed);
         uint32_t nz = 0;
 #pragma unroll
@@ -420,24 +651,32 @@ __device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint
             xr[v] &= ~P[v];
             nz |= xr[v];
         }
+        bool contra_lane = false;
         if (valid && !nz && nonzero4(yr)) {
-            ++cnt;
-            first = min(first, seen + i);
+            cnt += weight;
+            first = min(first, seen + (long long)i);
+            contra_lane = true;
         }
         const uint32_t cand = __ballot_sync(FULL, valid && nz != 0u);
-        if (lane == 0) candw[32 * par + warp] = cand;
-        __syncthreads();
-        uint32_t wmask = 0;
-        for (int ww = 0; ww < nwarps; ++ww)
-            if (candw[32 * par + ww]) wmask |= 1u << ww;
+        uint32_t wmask;
+        if (CTA) {
+            if (lane == 0) wc[warp] = cand;
+            __syncthreads();
+            wmask = 0;
+            for (int ww = 0; ww < G; ++ww)
+                if (wc[ww]) wmask |= 1u << ww;
+        } else {
+            wmask = cand ? 1u : 0u;
+        }
         if (wmask) {
             const int first_warp = __ffs(wmask) - 1;
             for (uint32_t wm = wmask; wm; wm &= wm - 1) {
                 const int ww = __ffs(wm) - 1;
                 if (warp == ww) {
-                    if (ww != first_warp) reduce_new<WD>(xr, yr, S, NPR);
+                    if (CTA && ww != first_warp) reduce_new<WD>(xr, yr, S, NPR);
                     uint32_t NP[WD];
-                    const int added = insert_block<WD>(xr, yr, cand, S, P, cd.d, lane, seen + i, first, cnt, NP);
+                    const int added = insert_block<WD>(xr, yr, cand, S, P, cd.d, lane, seen + (long long)i, first, cnt,
+                                                       NP, contra_lane, weight);
                     if (lane == 0 && added) {
 #pragma unroll
                         for (int v = 0; v < WD; ++v) {
@@ -447,20 +686,23 @@ __device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint
                         *rank_s += added;
                     }
                 }
-                __syncthreads();
+                group_sync<CTA>();
 #pragma unroll
                 for (int v = 0; v < WD; ++v) P[v] = Ps[v];
             }
             mixed = mixed_words<WD>(P, cd.d, cd.wd);
-            if (t < 48) NPR[t] = 0;
+            if (CTA) {
+                if (t < 48) NPR[t] = 0u;
+            }
         }
+        (void)contra_lane;
     }
     warp_stats(first, cnt);
     if (lane == 0 && cnt) {
         atomicAdd(cnt_s, cnt);
         atomicMin(first_s, first);
     }
-    __syncthreads();
+    group_sync<CTA>();
     if (t < cd.wd) s.pivot[cd.pw_off + t] = Ps[t];
     basis_from_smem<WD>(s, cd, S, t, nt);
     if (t == 0) {
@@ -468,7 +710,7 @@ __device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint
         s.rows_seen[c] = seen + T;
         commit_stats(s, c, *first_s, *cnt_s);
     }
-    __syncthreads();
+    group_sync<CTA>();
 }
 
 #define F2_NARROW_SWITCH(wd, CALL)   \
@@ -485,7 +727,7 @@ __device__ void learn_ctx_cta(const StoreDev& s, const LearnArgs& a, int c, uint
     default: break;                  \
     }
 
-__global__ void __launch_bounds__(LEARN_WARPS * 32) learn_narrow_kernel(StoreDev s, LearnArgs a)
+__global__ void __launch_bounds__(LEARN_WARPS * 32, 2) elim_narrow_kernel(StoreDev s, LearnArgs a)
 {
     extern __shared__ __align__(16) uint32_t smem[];
     __shared__ int s_item;
@@ -494,13 +736,13 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32) learn_narrow_kernel(StoreDev
     const int b_cta = a.counters[CNT_BEGIN + CLS_CTA];
     for (;;) {
         __syncthreads();
-        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD_CTA, 1);
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_CTA, 1);
         __syncthreads();
         const int item = s_item;
         if (item >= n_cta) break;
         const int c = a.queue[b_cta + item];
         const int wd = s.desc[c].wd;
-#define F2_CALL_CTA(W) learn_ctx_cta<W>(s, a, c, smem)
+#define F2_CALL_CTA(W) elim_ctx<W, true>(s, a, c, smem)
         F2_NARROW_SWITCH(wd, F2_CALL_CTA)
 #undef F2_CALL_CTA
     }
@@ -509,12 +751,12 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32) learn_narrow_kernel(StoreDev
     uint32_t* region = smem + warp * a.warp_region_words;
     for (;;) {
         int item = 0;
-        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD_WARP, 1);
+        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_WARP, 1);
         item = __shfl_sync(FULL, item, 0);
         if (item >= n_w) break;
         const int c = a.queue[b_w + item];
         const int wd = s.desc[c].wd;
-#define F2_CALL_WARP(W) learn_ctx_warp<W>(s, a, c, region, lane)
+#define F2_CALL_WARP(W) elim_ctx<W, false>(s, a, c, region)
         F2_NARROW_SWITCH(wd, F2_CALL_WARP)
 #undef F2_CALL_WARP
     }
@@ -522,7 +764,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32) learn_narrow_kernel(StoreDev
 
 constexpr int WIDE_WD = 33;
 
-__global__ void __launch_bounds__(WIDE_WARPS * 32) learn_wide_kernel(StoreDev s, LearnArgs a)
+__global__ void __launch_bounds__(WIDE_WARPS * 32) elim_wide_kernel(StoreDev s, LearnArgs a)
 {
     extern __shared__ __align__(16) uint32_t smem[];
     __shared__ int s_item;
@@ -530,42 +772,61 @@ __global__ void __launch_bounds__(WIDE_WARPS * 32) learn_wide_kernel(StoreDev s,
     const int b = a.counters[CNT_BEGIN + CLS_WIDE];
     for (;;) {
         __syncthreads();
-        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD_WIDE, 1);
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_WIDE, 1);
         __syncthreads();
         const int item = s_item;
         if (item >= n) break;
-        learn_ctx_cta<WIDE_WD>(s, a, a.queue[b + item], smem);
+        elim_ctx<WIDE_WD, true>(s, a, a.queue[b + item], smem);
     }
 }
 
-// Validate the batch and build the longest-first queues (one block).
+// Validate the batch and order the work longest-first (one block).
+//   mode 0 (dedup plan): every valid non-empty context goes to the warp or
+//     CTA dedup queue by its row count; rep_count[c] is set to -1 for an
+//     invalid context and 0 for an empty one (the dedup pass fills the rest);
+//   mode 1 (elimination plan): contexts with representatives (rep_count, or
+//     all rows when rep_count is NULL, after the same validation) go to the
+//     warp, CTA or wide elimination queue.
 __global__ void __launch_bounds__(1024) plan_kernel(StoreDev s, const int64_t* __restrict__ row_off,
                                                     const int64_t* __restrict__ x_off, int64_t total_rows,
-                                                    int64_t total_xw, int warp_region_words, int64_t heavy_rows,
+                                                    int64_t total_xw, int32_t* __restrict__ rep_count, int mode,
+                                                    int warp_region_words, int64_t heavy_rows, int64_t warp_work,
                                                     int32_t* __restrict__ queue, int32_t* __restrict__ keybuf,
                                                     int* __restrict__ counters)
 {
-    __shared__ int hist[3][PLAN_BUCKETS];
-    __shared__ int cursor[3][PLAN_BUCKETS];
-    for (int i = threadIdx.x; i < 3 * PLAN_BUCKETS; i += blockDim.x) (&hist[0][0])[i] = 0;
+    __shared__ int hist[NUM_CLASSES][PLAN_BUCKETS];
+    __shared__ int cursor[NUM_CLASSES][PLAN_BUCKETS];
+    for (int i = threadIdx.x; i < NUM_CLASSES * PLAN_BUCKETS; i += blockDim.x) (&hist[0][0])[i] = 0;
     __syncthreads();
     for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
         const CtxDesc cd = s.desc[c];
-        const int64_t a0 = row_off[c], a1 = row_off[c + 1];
-        const int64_t rows = a1 - a0;
-        const int64_t x0 = x_off[c];
-        const bool ok = a0 >= 0 && rows >= 0 && a1 <= total_rows && x0 >= 0 && rows <= total_xw &&
-                        x0 + rows * cd.xw <= total_xw;
+        int64_t R;
+        if (mode == 1 && rep_count) {
+            R = rep_count[c];
+        } else {
+            const int64_t a0 = row_off[c], a1 = row_off[c + 1];
+            const int64_t rows = a1 - a0;
+            const int64_t x0 = x_off[c];
+            const bool ok = a0 >= 0 && rows >= 0 && rows < (1ll << 31) && a1 <= total_rows && x0 >= 0 &&
+                            rows <= total_xw && x0 + rows * cd.xw <= total_xw;
+            if (!ok) record_status(s.status, F2_ERR_ROWS);
+            R = ok ? rows : -1;
+            if (mode == 0 && rep_count) rep_count[c] = (R > 0) ? 0 : (int32_t)R;
+        }
         int key = -1;
-        if (!ok) {
-            record_status(s.status, F2_ERR_ROWS);
-        } else if (rows > 0) {
-            const int basis_words = WARP_CTL + cd.d * row_stride(cd.wd);
+        if (R > 0) {
             int cls;
-            if (cd.wd > NARROW_WD) cls = CLS_WIDE;
-            else if (basis_words > warp_region_words || rows >= heavy_rows) cls = CLS_CTA;
-            else cls = CLS_WARP;
-            const unsigned long long work = (unsigned long long)rows * (unsigned long long)(cd.wd + 4);
+            unsigned long long work;
+            if (mode == 0) {
+                cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : CLS_DD_CTA;
+                work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
+            } else {
+                if (cd.wd > NARROW_WD) cls = CLS_WIDE;
+                else if (elim_words(cd.d, cd.wd) > warp_region_words || R >= heavy_rows || R * cd.d > warp_work)
+                    cls = CLS_CTA;
+                else cls = CLS_WARP;
+                work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
+            }
             int bucket = 63 - __clzll(work);
             if (bucket >= PLAN_BUCKETS) bucket = PLAN_BUCKETS - 1;
             key = cls * PLAN_BUCKETS + bucket;
@@ -576,17 +837,15 @@ __global__ void __launch_bounds__(1024) plan_kernel(StoreDev s, const int64_t* _
     __syncthreads();
     if (threadIdx.x == 0) {
         int pos = 0;
-        for (int cls = 0; cls < 3; ++cls) {
+        for (int cls = 0; cls < NUM_CLASSES; ++cls) {
             counters[CNT_BEGIN + cls] = pos;
             for (int bk = PLAN_BUCKETS - 1; bk >= 0; --bk) {
                 cursor[cls][bk] = pos;
                 pos += hist[cls][bk];
             }
             counters[CNT_COUNT + cls] = pos - counters[CNT_BEGIN + cls];
+            counters[CNT_HEAD + cls] = 0;
         }
-        counters[CNT_HEAD_CTA] = 0;
-        counters[CNT_HEAD_WIDE] = 0;
-        counters[CNT_HEAD_WARP] = 0;
     }
     __syncthreads();
     for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
@@ -600,6 +859,68 @@ __global__ void __launch_bounds__(1024) plan_kernel(StoreDev s, const int64_t* _
 
 inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) == 0; }
 
+// Shared-memory need of the narrow elimination kernel for a set of widths.
+size_t narrow_smem(int max_narrow_words, int warp_region_words)
+{
+    const size_t cta = 4 * (size_t)max_narrow_words;
+    const size_t warps = 4 * (size_t)LEARN_WARPS * (size_t)warp_region_words;
+    return cta > warps ? cta : warps;
+}
+
+// Enqueue pass 2 (plan + kernels) for one batch.
+int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* row_off, const int64_t* x_off,
+                       int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
+                       int64_t warp_work, int32_t* queue, int32_t* keybuf, int num_sms, int max_narrow_words,
+                       bool has_narrow, int max_wide_d, bool has_wide, cudaStream_t cs)
+{
+    plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off, x_off, total_rows, total_xw, rep_count, 1, la.warp_region_words,
+                                    heavy_rows, warp_work, queue, keybuf, la.counters);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    if (has_narrow) {
+        const size_t smem = narrow_smem(max_narrow_words, la.warp_region_words);
+        e = cudaFuncSetAttribute(elim_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        int per_sm = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, elim_narrow_kernel, LEARN_WARPS * 32, smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        if (per_sm < 1) per_sm = 1;
+        elim_narrow_kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    if (has_wide) {
+        const size_t smem = 4 * (size_t)elim_words(max_wide_d, WIDE_WD);
+        e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, cs>>>(sd, la);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    return F2_OK;
+}
+
+// Widest narrow basis (words of an elimination group) and widest row.
+void width_summary(const int32_t* n_bits, int32_t num_ctx, bool raw, int* max_narrow_words, bool* has_narrow,
+                   int* max_wide_d, bool* has_wide)
+{
+    *max_narrow_words = 0;
+    *max_wide_d = 0;
+    *has_narrow = *has_wide = false;
+    for (int32_t c = 0; c < num_ctx; ++c) {
+        const int d = raw ? n_bits[c] : n_bits[c] + 1;
+        const int wd = (d + 31) / 32;
+        if (wd <= NARROW_WD) {
+            *has_narrow = true;
+            const int w = elim_words(d, wd);
+            if (w > *max_narrow_words) *max_narrow_words = w;
+        } else {
+            *has_wide = true;
+            if (d > *max_wide_d) *max_wide_d = d;
+        }
+    }
+}
+
 }  // namespace
 
 extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint32_t* x, const int64_t* x_off,
@@ -612,57 +933,58 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     if (!is_aligned(row_off, 8) || !is_aligned(x_off, 8) || !is_aligned(x, 4) || !is_aligned(y, 16))
         return F2_ERR_ALIGN;
     cudaStream_t cs = (cudaStream_t)stream;
+    cudaError_t e;
+    const bool dedup = st->dedup && total_rows > 0;
+    if (dedup && total_rows > st->rep_capacity) {  // per-row scratch of pass 1, grown stream-ordered
+        if (st->rep_list) cudaFreeAsync(st->rep_list, cs);
+        if (st->rep_dup) cudaFreeAsync(st->rep_dup, cs);
+        st->rep_list = st->rep_dup = nullptr;
+        st->rep_capacity = 0;
+        e = cudaMallocAsync((void**)&st->rep_list, sizeof(int32_t) * (size_t)total_rows, cs);
+        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->rep_dup, sizeof(int32_t) * (size_t)total_rows, cs);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        st->rep_capacity = total_rows;
+    }
     const StoreDev sd = st->dev();
-    const int warp_region_words = (int)(st->warp_basis_bytes / 4);
-    plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off, x_off, total_rows, total_x_words, warp_region_words,
-                                    st->heavy_rows, st->queue, st->keybuf, st->counters);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return f2_cuda_status(e);
-
+    if (dedup) {
+        plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off, x_off, total_rows, total_x_words, st->rep_count, 0, 0, 0, 0,
+                                        st->queue, st->keybuf, st->counters);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        DedupArgs da;
+        da.row_off = row_off;
+        da.x_off = x_off;
+        da.x = x;
+        da.y = reinterpret_cast<const uint4*>(y);
+        da.rep_list = st->rep_list;
+        da.rep_dup = st->rep_dup;
+        da.rep_count = st->rep_count;
+        da.queue = st->queue;
+        da.counters = st->counters;
+        e = cudaFuncSetAttribute(dedup_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        dedup_kernel<<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
     LearnArgs la;
     la.row_off = row_off;
     la.x_off = x_off;
     la.x = x;
     la.y = reinterpret_cast<const uint4*>(y);
+    la.rep_list = dedup ? st->rep_list : nullptr;
+    la.rep_dup = dedup ? st->rep_dup : nullptr;
+    la.rep_count = dedup ? st->rep_count : nullptr;
     la.queue = st->queue;
     la.counters = st->counters;
-    la.warp_region_words = warp_region_words;
-
-    // narrow kernel: CTA-mode contexts first (largest basis of any narrow
-    // context), then the warp queue (LEARN_WARPS regions)
-    int max_narrow_d = 0, max_narrow_wd = 1;
-    for (int32_t c = 0; c < st->num_ctx; ++c) {
-        const int d = (st->flags & F2_FLAG_RAW_FEATURES) ? st->n_bits[(size_t)c] : st->n_bits[(size_t)c] + 1;
-        const int wd = (d + 31) / 32;
-        if (wd <= NARROW_WD && d * row_stride(wd) > max_narrow_d * row_stride(max_narrow_wd)) {
-            max_narrow_d = d;
-            max_narrow_wd = wd;
-        }
-    }
-    if (st->n_wide < st->num_ctx) {
-        size_t cta_bytes = 4 * (size_t)(CTL_WORDS + max_narrow_d * row_stride(max_narrow_wd));
-        size_t warp_bytes = 4 * (size_t)LEARN_WARPS * (size_t)warp_region_words;
-        size_t smem = cta_bytes > warp_bytes ? cta_bytes : warp_bytes;
-        e = cudaFuncSetAttribute(learn_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        int per_sm = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, learn_narrow_kernel, LEARN_WARPS * 32, smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        if (per_sm < 1) per_sm = 1;
-        learn_narrow_kernel<<<st->num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
-    }
-    if (st->n_wide > 0) {
-        const size_t smem = 4 * (size_t)(CTL_WORDS + st->max_d * row_stride(WIDE_WD));
-        e = cudaFuncSetAttribute(learn_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        int blocks = st->n_wide < st->num_sms ? st->n_wide : st->num_sms;
-        learn_wide_kernel<<<blocks, WIDE_WARPS * 32, smem, cs>>>(sd, la);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
-    }
-    return F2_OK;
+    la.warp_region_words = (int)(st->warp_basis_bytes / 4);
+    int max_narrow_words, max_wide_d;
+    bool has_narrow, has_wide;
+    width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0, &max_narrow_words,
+                  &has_narrow, &max_wide_d, &has_wide);
+    return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
+                              st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->num_sms, max_narrow_words,
+                              has_narrow, max_wide_d, has_wide, cs);
 }
 
 // ---------------------------------------------------------------------------
@@ -679,7 +1001,7 @@ struct NoallocScratch {
     int32_t n_bits[F2_NOALLOC_MAX_CTX];
     int32_t queue[F2_NOALLOC_MAX_CTX];
     int32_t keybuf[F2_NOALLOC_MAX_CTX];
-    int counters[16];
+    int counters[32];
 };
 
 // Device storage for the scratch; in host code this name is only a symbol
@@ -687,9 +1009,8 @@ struct NoallocScratch {
 static __device__ __align__(256) unsigned char g_noalloc_scratch[sizeof(NoallocScratch)];
 
 constexpr int NOALLOC_MAX_DEVICES = 64;
-constexpr int NOALLOC_NARROW_SMEM_DEFAULT = 4 * LEARN_WARPS * (8192 / 4);
-constexpr int NOALLOC_HEAVY_ROWS = 4096;
-constexpr int NOALLOC_WARP_REGION_WORDS = 8192 / 4;
+constexpr int NOALLOC_HEAVY_ROWS = DEFAULT_HEAVY_ROWS;
+constexpr int NOALLOC_WARP_REGION_WORDS = DEFAULT_WARP_REGION_BYTES / 4;
 
 struct NoallocDevice {
     NoallocScratch* scratch;
@@ -822,21 +1143,8 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
         !is_aligned(basis_x_dev, 4) || !is_aligned(status_dev, 4))
         return F2_ERR_ALIGN;
     const bool raw = (flags & F2_FLAG_RAW_FEATURES) != 0;
-    int max_narrow_bytes = 0, max_d = 0, n_wide = 0, n_narrow = 0;
-    for (int32_t c = 0; c < num_ctx; ++c) {
-        const int n = n_bits_host[c];
-        if (n < 1 || n > MAX_N) return F2_ERR_NBITS;
-        const int d = raw ? n : n + 1;
-        const int wd = (d + 31) / 32;
-        if (d > max_d) max_d = d;
-        if (wd > NARROW_WD) {
-            ++n_wide;
-        } else {
-            ++n_narrow;
-            const int bytes = 4 * (CTL_WORDS + d * row_stride(wd));
-            if (bytes > max_narrow_bytes) max_narrow_bytes = bytes;
-        }
-    }
+    for (int32_t c = 0; c < num_ctx; ++c)
+        if (n_bits_host[c] < 1 || n_bits_host[c] > MAX_N) return F2_ERR_NBITS;
     NoallocDevice* nd = nullptr;
     int rc = noalloc_setup(&nd);
     if (rc != F2_OK) return rc;
@@ -862,39 +1170,21 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     sd.status = status_dev;
     sd.num_ctx = num_ctx;
     sd.raw = raw ? 1u : 0u;
-    plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off_dev, x_off_dev, total_rows, total_x_words, NOALLOC_WARP_REGION_WORDS,
-                                    NOALLOC_HEAVY_ROWS, sc->queue, sc->keybuf, sc->counters);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return f2_cuda_status(e);
-
     LearnArgs la;
     la.row_off = row_off_dev;
     la.x_off = x_off_dev;
     la.x = x_dev;
     la.y = reinterpret_cast<const uint4*>(y_dev);
+    la.rep_list = nullptr;  // every row is its own representative: no per-row scratch
+    la.rep_dup = nullptr;
+    la.rep_count = nullptr;
     la.queue = sc->queue;
     la.counters = sc->counters;
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
-    if (n_narrow) {
-        const int smem = max_narrow_bytes > NOALLOC_NARROW_SMEM_DEFAULT ? max_narrow_bytes : NOALLOC_NARROW_SMEM_DEFAULT;
-        e = cudaFuncSetAttribute(learn_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        int per_sm = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, learn_narrow_kernel, LEARN_WARPS * 32, smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        if (per_sm < 1) per_sm = 1;
-        learn_narrow_kernel<<<nd->num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
-    }
-    if (n_wide) {
-        const int smem = 4 * (CTL_WORDS + max_d * row_stride(WIDE_WD));
-        e = cudaFuncSetAttribute(learn_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        const int blocks = n_wide < nd->num_sms ? n_wide : nd->num_sms;
-        learn_wide_kernel<<<blocks, WIDE_WARPS * 32, smem, cs>>>(sd, la);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
-    }
-    return F2_OK;
+    int max_narrow_words, max_wide_d;
+    bool has_narrow, has_wide;
+    width_summary(n_bits_host, num_ctx, raw, &max_narrow_words, &has_narrow, &max_wide_d, &has_wide);
+    return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,
+                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, nd->num_sms, max_narrow_words, has_narrow,
+                              max_wide_d, has_wide, cs);
 }

@@ -37,8 +37,9 @@ extern "C" const char* f2_status_string(int status)
 static void free_store(f2_store* s)
 {
     if (!s) return;
-    void* ptrs[] = {s->desc, s->rank, s->contra, s->first_contra, s->n_contra, s->rows_seen, s->pivot,
-                    s->bx, s->bz, s->status, s->queue, s->keybuf, s->counters};
+    void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
+                    s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
+                    s->counters, s->rep_count, s->rep_list, s->rep_dup};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     delete s;
@@ -76,8 +77,10 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     if (!s) return F2_ERR_OOM;
     s->num_ctx = num_ctx;
     s->flags = flags;
-    s->heavy_rows = 4096;
-    s->warp_basis_bytes = 8192;
+    s->heavy_rows = DEFAULT_HEAVY_ROWS;
+    s->warp_basis_bytes = DEFAULT_WARP_REGION_BYTES;
+    s->warp_work = DEFAULT_WARP_WORK;
+    s->dedup = 1;
     if (cudaGetDevice(&s->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
         delete s;
@@ -127,7 +130,8 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     alloc((void**)&s->status, sizeof(int));
     alloc((void**)&s->queue, sizeof(int32_t) * C);
     alloc((void**)&s->keybuf, sizeof(int32_t) * C);
-    alloc((void**)&s->counters, sizeof(int) * 16);
+    alloc((void**)&s->counters, sizeof(int) * CNT_WORDS);
+    alloc((void**)&s->rep_count, sizeof(int32_t) * C);
     cudaStream_t st = (cudaStream_t)stream;
     if (e == cudaSuccess && num_ctx)
         e = cudaMemcpyAsync(s->desc, desc.data(), sizeof(CtxDesc) * (size_t)num_ctx,
@@ -356,6 +360,14 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_WARP_BASIS_BYTES:
         if (value < 0 || value > 24576) return F2_ERR_INVALID_ARG;
         s->warp_basis_bytes = (value / 16) * 16;
+        return F2_OK;
+    case F2_OPT_WARP_WORK:
+        if (value < 0) return F2_ERR_INVALID_ARG;
+        s->warp_work = value;
+        return F2_OK;
+    case F2_OPT_DEDUP:
+        if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
+        s->dedup = (int)value;
         return F2_OK;
     default:
         return F2_ERR_INVALID_ARG;

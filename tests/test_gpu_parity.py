@@ -157,6 +157,7 @@ def test_config2_scaled(env, mode):
         st.set_option(binding.F2_OPT_HEAVY_ROWS, 1)
     if mode == "all_warp":
         st.set_option(binding.F2_OPT_HEAVY_ROWS, 1 << 40)
+        st.set_option(binding.F2_OPT_WARP_WORK, 1 << 50)
         st.set_option(binding.F2_OPT_WARP_BASIS_BYTES, 24576)
     gpu_learn_workload(binding, st, wl, dev)
     O = oracle_for(wl)
