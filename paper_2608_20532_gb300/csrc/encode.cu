@@ -43,18 +43,36 @@ __device__ __forceinline__ bool encode_one(const StoreDev& s, const CtxDesc& cd,
         if (w < cd.wd) {
             const uint32_t pw = __ldg(P + w);
             uint32_t m = q[w] & pw;
+            // up to four stored rows per step: their loads are independent, so
+            // they are issued together before any XOR
+            constexpr int U = (WD <= NARROW_WD) ? 4 : 1;
             while (m) {
-                const int b = __ffs(m) - 1;
-                m &= m - 1;
-                const int k = 32 * w + b;
-                const uint4 z = __ldg(Z + k);
-                acc.x ^= z.x;
-                acc.y ^= z.y;
-                acc.z ^= z.z;
-                acc.w ^= z.w;
-                const uint32_t* rk = X + (int64_t)k * cd.wd;
+                int k[U];
+                bool use[U];
 #pragma unroll
-                for (int v = 0; v <= w; ++v) q[v] ^= __ldg(rk + v);
+                for (int u = 0; u < U; ++u) {
+                    use[u] = m != 0u;
+                    k[u] = use[u] ? 32 * w + __ffs(m) - 1 : 0;
+                    m &= m - 1;
+                }
+                uint4 z[U];
+                uint32_t xv[U][WD];
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    z[u] = use[u] ? __ldg(Z + k[u]) : make_uint4(0, 0, 0, 0);
+                    const uint32_t* rk = X + (int64_t)k[u] * cd.wd;
+#pragma unroll
+                    for (int v = 0; v <= w; ++v) xv[u][v] = use[u] ? __ldg(rk + v) : 0u;
+                }
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    acc.x ^= z[u].x;
+                    acc.y ^= z[u].y;
+                    acc.z ^= z[u].z;
+                    acc.w ^= z[u].w;
+#pragma unroll
+                    for (int v = 0; v <= w; ++v) q[v] ^= xv[u][v];
+                }
             }
         }
     }
@@ -67,7 +85,7 @@ __device__ __forceinline__ bool encode_one(const StoreDev& s, const CtxDesc& cd,
     return resid == 0;
 }
 
-__global__ void __launch_bounds__(256) encode_kernel(StoreDev s, int64_t Q, const int32_t* __restrict__ ctx_id,
+__global__ void __launch_bounds__(256, 3) encode_kernel(StoreDev s, int64_t Q, const int32_t* __restrict__ ctx_id,
                                                      const uint32_t* __restrict__ x, int stride,
                                                      uint4* __restrict__ y, uint8_t* __restrict__ in_span)
 {

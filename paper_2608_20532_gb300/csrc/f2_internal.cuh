@@ -29,8 +29,16 @@ enum Counter {
     CNT_WORDS = 32
 };
 // Work classes: elimination by a CTA / the wide kernel / a warp, and dedup
-// by a CTA / a warp.
-enum Class { CLS_CTA = 0, CLS_WIDE = 1, CLS_WARP = 2, CLS_DD_CTA = 3, CLS_DD_WARP = 4, NUM_CLASSES = 5 };
+// by a CTA / a quad of warps / a warp.
+enum Class {
+    CLS_CTA = 0,
+    CLS_WIDE = 1,
+    CLS_WARP = 2,
+    CLS_DD_CTA = 3,
+    CLS_DD_QUAD = 4,
+    CLS_DD_WARP = 5,
+    NUM_CLASSES = 6
+};
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {
@@ -103,6 +111,7 @@ struct f2_store {
     int32_t* queue;
     int32_t* keybuf;
     int* counters;
+    int* plan_hist;         // key histogram / cursors of the plan kernels
     int32_t* rep_count;     // representatives per context (pass 1 output)
     int32_t* rep_list;      // per-row scratch of pass 1 (capacity rep_capacity rows)
     int32_t* rep_dup;

@@ -85,16 +85,35 @@ constexpr int CTL_WORDS = 176; // size of the control area (16-byte multiple)
 // (fingerprint, row index) plus a duplicate counter: 12 bytes.
 constexpr int DD_THREADS = 512;
 constexpr int DD_WARPS = DD_THREADS / 32;
-constexpr int DD_WARP_MAX_ROWS = 512;
+constexpr int DD_WARP_MAX_ROWS = 512;           // warp-owned up to this many rows
+constexpr int DD_QUAD_MAX_ROWS = 8192;          // 4-warp-owned up to this many rows
 constexpr int DD_WARP_E = 1024;
 constexpr int DD_WARP_REGION = 3 * DD_WARP_E;   // words
+constexpr int DD_QUAD_E = 4 * DD_WARP_E;
 constexpr int DD_CTA_E = 16384;
 constexpr int DD_SMEM = 4 * 3 * DD_CTA_E;       // bytes (also 16 warp regions)
 constexpr int DD_K = 4;                         // rows per thread in flight
+constexpr int DD_XW = NARROW_WD;                // widest feature row (words) that is deduplicated
 constexpr int DEDUP_PROBES = 8;                 // linear-probe limit
 static_assert(DD_WARPS * DD_WARP_REGION * 4 <= DD_SMEM, "warp regions exceed the dedup shared memory");
 
 __host__ __device__ __forceinline__ int elim_words(int d, int wd) { return CTL_WORDS + d * row_stride(wd); }
+
+// Dispatch on a width 1..9 (feature words) to a template instantiation.
+#define F2_NARROW_SWITCH(wd, CALL)   \
+    switch (wd) {                    \
+    case 1: CALL(1); break;          \
+    case 2: CALL(2); break;          \
+    case 3: CALL(3); break;          \
+    case 4: CALL(4); break;          \
+    case 5: CALL(5); break;          \
+    case 6: CALL(6); break;          \
+    case 7: CALL(7); break;          \
+    case 8: CALL(8); break;          \
+    case 9: CALL(9); break;          \
+    default: break;                  \
+    }
+
 
 __device__ __forceinline__ bool nonzero4(const uint4& v) { return (v.x | v.y | v.z | v.w) != 0u; }
 
@@ -208,17 +227,16 @@ __device__ __forceinline__ bool rows_equal(const uint32_t* __restrict__ xc, cons
     return true;
 }
 
-// Find the entry of row i's content, inserting it if absent.  Returns the
-// slot (whose index field ends as the smallest row index of that content), or
-// -1 when the probe limit is reached (the row then counts as its own
-// representative, which is always exact).
-__device__ __forceinline__ int dd_find_insert(uint2* tab, int E, uint32_t h, int64_t i, const uint4& yi,
-                                              const uint32_t* __restrict__ xc, const uint4* __restrict__ yc, int xw,
-                                              int n)
+// Find the entry of row i's content starting at slot `slot`, inserting it
+// if absent.  Returns the slot (whose index field ends as the smallest row
+// index of that content), or -1 when the probe budget runs out (the row then
+// counts as its own representative, which is always exact).
+__device__ __noinline__ int dd_find_insert(uint2* tab, int E, uint32_t h, int64_t i, const uint4& yi,
+                                           const uint32_t* __restrict__ xc, const uint4* __restrict__ yc, int xw,
+                                           int n, uint32_t slot, int budget)
 {
     const uint32_t fp = h | 1u;
-    uint32_t slot = (h >> 7) & (uint32_t)(E - 1);
-    for (int p = 0; p < DEDUP_PROBES; ++p, slot = (slot + 1) & (uint32_t)(E - 1)) {
+    for (int p = 0; p < budget; ++p, slot = (slot + 1) & (uint32_t)(E - 1)) {
         uint2 e = tab[slot];
         if (e.x == 0u) {
             const unsigned long long want = ((unsigned long long)(uint32_t)i << 32) | fp;
@@ -235,90 +253,164 @@ __device__ __forceinline__ int dd_find_insert(uint2* tab, int E, uint32_t h, int
     return -1;
 }
 
-// One group (a warp, or the whole CTA) finds the representatives of context
-// c and writes them, in stream order, to rep_list[row_off[c] + k] with their
-// duplicate counts in rep_dup; rep_count[c] = number of representatives.
-template <bool CTA>
+// Group synchronisation for pass 1: a warp, a quad of 4 warps (named
+// barrier 1 + quad index, 128 threads) or the whole CTA.
+template <int G>
+__device__ __forceinline__ void dd_sync()
+{
+    if (G == 1) __syncwarp();
+    else if (G == DD_WARPS) __syncthreads();
+    else asm volatile("bar.sync %0, %1;" ::"r"(1 + (int)(threadIdx.x >> 5) / G), "r"(32 * G) : "memory");
+}
+
+// One group of G warps finds the representatives of context c and writes
+// them, in stream order, to rep_list[row_off[c] + k] with their duplicate
+// counts in rep_dup; rep_count[c] = number of representatives.  Each thread
+// keeps DD_K rows in flight.  Table slot: (fingerprint, smallest row index
+// of that content) plus a duplicate counter; a full row comparison decides
+// every match, so a row is a duplicate only if it equals an earlier row.
+template <int G, int XW>
 __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t* region, int E, int* wcnt)
 {
-    const int G = CTA ? (int)(blockDim.x >> 5) : 1;
+    constexpr int NT = 32 * G;
     const int lane = threadIdx.x & 31;
-    const int warp = CTA ? (int)(threadIdx.x >> 5) : 0;
-    const int t = 32 * warp + lane;
-    const int nt = 32 * G;
+    const int gw = (G == 1) ? 0 : (int)((threadIdx.x >> 5) % G);  // warp within the group
+    const int t = 32 * gw + lane;
     uint2* tab = reinterpret_cast<uint2*>(region);
     int* D = reinterpret_cast<int*>(region + 2 * E);
     const CtxDesc cd = s.desc[c];
-    const int xw = cd.xw, n = cd.n;
+    constexpr int xw = XW;
+    const int n = cd.n;
     const int64_t r0 = a.row_off[c];
     const int T = (int)(a.row_off[c + 1] - r0);
     const uint32_t* xc = a.x + a.x_off[c];
     const uint4* yc = a.y + r0;
     const uint32_t lm = last_mask(n);
-    for (int e = t; e < E; e += nt) {
+    const uint32_t emask = (uint32_t)(E - 1);
+    for (int e = t; e < E; e += NT) {
         tab[e] = make_uint2(0u, 0u);
         D[e] = 0;
     }
-    group_sync<CTA>();
+    dd_sync<G>();
     int nrep = 0;
-    for (int base = 0; base < T; base += nt * DD_K) {
+    for (int base = 0; base < T; base += NT * DD_K) {
         int mine[DD_K];
         uint32_t h[DD_K];
         uint4 yv[DD_K];
+        uint32_t xv[DD_K][XW];
+        // every load of the round first
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
-            const int i = base + j * nt + t;
-            h[j] = 0x811C9DC5u;
-            yv[j] = make_uint4(0, 0, 0, 0);
-            if (i < T) {
-                yv[j] = __ldg(yc + i);
-                for (int v = 0; v < xw; ++v)
-                    h[j] = fnv_step(h[j], __ldg(xc + (int64_t)i * xw + v) & ((v == xw - 1) ? lm : 0xffffffffu));
-                h[j] = fnv_step(fnv_step(fnv_step(fnv_step(h[j], yv[j].x), yv[j].y), yv[j].z), yv[j].w);
-                h[j] = fmix32(h[j]);
+            const int i = base + j * NT + t;
+            const bool ok = i < T;
+            yv[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int v = 0; v < XW; ++v) {
+                uint32_t w = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
+                if (v == XW - 1) w &= lm;
+                xv[j][v] = w;
             }
         }
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
-            const int i = base + j * nt + t;
-            mine[j] = (i < T) ? dd_find_insert(tab, E, h[j], i, yv[j], xc, yc, xw, n) : -1;
+            uint32_t hh = 0x811C9DC5u;
+#pragma unroll
+            for (int v = 0; v < XW; ++v) hh = fnv_step(hh, xv[j][v]);
+            h[j] = fmix32(fnv_step(fnv_step(fnv_step(fnv_step(hh, yv[j].x), yv[j].y), yv[j].z), yv[j].w));
         }
-        group_sync<CTA>();
+        // home slots (shared memory)
+        uint2 ent[DD_K];
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
-            const int i = base + j * nt + t;
+            const int i = base + j * NT + t;
+            mine[j] = (i < T) ? -2 : -1;  // -2 = unresolved
+            ent[j] = make_uint2(0u, 0u);
+            if (i < T) {
+                const uint32_t slot = (h[j] >> 7) & emask;
+                ent[j] = tab[slot];
+                if (ent[j].x == 0u) {
+                    const unsigned long long want = ((unsigned long long)(uint32_t)i << 32) | (h[j] | 1u);
+                    const unsigned long long old =
+                        atomicCAS(reinterpret_cast<unsigned long long*>(tab + slot), 0ull, want);
+                    if (old == 0ull) {
+                        mine[j] = (int)slot;
+                    } else {
+                        ent[j].x = (uint32_t)old;
+                        ent[j].y = (uint32_t)(old >> 32);
+                    }
+                }
+            }
+        }
+        // full comparison with the matching rows (loads issued together)
+        bool eq[DD_K];
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            eq[j] = false;
+            if (mine[j] == -2 && ent[j].x == (h[j] | 1u)) {
+                const int64_t o = ent[j].y;
+                const uint4 yo = __ldg(yc + o);
+                bool e = yo.x == yv[j].x && yo.y == yv[j].y && yo.z == yv[j].z && yo.w == yv[j].w;
+#pragma unroll
+                for (int v = 0; v < XW; ++v) {
+                    uint32_t w = __ldg(xc + o * XW + v);
+                    if (v == XW - 1) w &= lm;
+                    e = e && (w == xv[j][v]);
+                }
+                eq[j] = e;
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            if (mine[j] != -2) continue;
+            const int i = base + j * NT + t;
+            const uint32_t slot = (h[j] >> 7) & emask;
+            if (eq[j]) {
+                if ((uint32_t)i < ent[j].y) atomicMin(&tab[slot].y, (uint32_t)i);
+                mine[j] = (int)slot;
+            } else {  // slow path: keep probing
+                mine[j] = dd_find_insert(tab, E, h[j], i, yv[j], xc, yc, xw, n, (slot + 1) & emask, DEDUP_PROBES - 1);
+            }
+        }
+        dd_sync<G>();
+        uint32_t bal[DD_K];
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            const int i = base + j * NT + t;
             const bool valid = i < T;
             const int rep = (valid && mine[j] >= 0) ? (int)tab[mine[j]].y : i;
             const bool isrep = valid && rep == i;
             if (valid && !isrep) atomicAdd(D + mine[j], 1);
-            const uint32_t bal = __ballot_sync(FULL, isrep);
-            int before = 0, total = __popc(bal);
-            if (CTA) {
-                if (lane == 0) wcnt[warp] = total;
-                __syncthreads();
+            bal[j] = __ballot_sync(FULL, isrep);
+            if (G > 1 && lane == 0) wcnt[gw * DD_K + j] = __popc(bal[j]);
+        }
+        if (G > 1) dd_sync<G>();
+#pragma unroll
+        for (int j = 0; j < DD_K; ++j) {
+            int before = 0, total = __popc(bal[j]);
+            if (G > 1) {
                 total = 0;
                 for (int ww = 0; ww < G; ++ww) {
-                    const int v = wcnt[ww];
-                    if (ww < warp) before += v;
+                    const int v = wcnt[ww * DD_K + j];
+                    if (ww < gw) before += v;
                     total += v;
                 }
-                __syncthreads();
             }
-            if (isrep) {
-                const int pos = nrep + before + __popc(bal & ((1u << lane) - 1u));
-                a.rep_list[r0 + pos] = i;
+            if ((bal[j] >> lane) & 1u) {
+                const int pos = nrep + before + __popc(bal[j] & ((1u << lane) - 1u));
+                a.rep_list[r0 + pos] = base + j * NT + t;
                 a.rep_dup[r0 + pos] = mine[j];
             }
             nrep += total;
         }
+        if (G > 1) dd_sync<G>();
     }
-    group_sync<CTA>();
-    for (int k = t; k < nrep; k += nt) {
+    dd_sync<G>();
+    for (int k = t; k < nrep; k += NT) {
         const int slot = a.rep_dup[r0 + k];
         a.rep_dup[r0 + k] = (slot >= 0) ? D[slot] : 0;
     }
     if (t == 0) a.rep_count[c] = nrep;
-    group_sync<CTA>();
+    dd_sync<G>();
 }
 
 __device__ __forceinline__ int pow2_at_least(int v)
@@ -328,37 +420,67 @@ __device__ __forceinline__ int pow2_at_least(int v)
     return e;
 }
 
+// Pass 1 kernel: CTA-owned contexts first, then quads, then warps.
 __global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupArgs a)
 {
     extern __shared__ __align__(16) uint32_t smem[];
-    __shared__ int s_item;
-    __shared__ int wcnt[32];
+    __shared__ int s_item[DD_WARPS];
+    __shared__ int wcnt[DD_WARPS * DD_K];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_cta = a.counters[CNT_COUNT + CLS_DD_CTA];
-    const int b_cta = a.counters[CNT_BEGIN + CLS_DD_CTA];
-    for (;;) {
-        __syncthreads();
-        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_CTA, 1);
-        __syncthreads();
-        const int item = s_item;
-        if (item >= n_cta) break;
-        const int c = a.queue[b_cta + item];
-        const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
-        int E = pow2_at_least(2 * T);
-        if (E > DD_CTA_E) E = DD_CTA_E;
-        dedup_ctx<true>(s, a, c, smem, E, wcnt);
+    {
+        const int n = a.counters[CNT_COUNT + CLS_DD_CTA];
+        const int b = a.counters[CNT_BEGIN + CLS_DD_CTA];
+        for (;;) {
+            __syncthreads();
+            if (threadIdx.x == 0) s_item[0] = atomicAdd(a.counters + CNT_HEAD + CLS_DD_CTA, 1);
+            __syncthreads();
+            const int item = s_item[0];
+            if (item >= n) break;
+            const int c = a.queue[b + item];
+            const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
+            int E = pow2_at_least(2 * T);
+            if (E > DD_CTA_E) E = DD_CTA_E;
+#define F2_DD_CTA(W) dedup_ctx<DD_WARPS, W>(s, a, c, smem, E, wcnt)
+            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_CTA)
+#undef F2_DD_CTA
+        }
     }
-    const int n_w = a.counters[CNT_COUNT + CLS_DD_WARP];
-    const int b_w = a.counters[CNT_BEGIN + CLS_DD_WARP];
-    uint32_t* region = smem + warp * DD_WARP_REGION;
-    for (;;) {
-        int item = 0;
-        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_WARP, 1);
-        item = __shfl_sync(FULL, item, 0);
-        if (item >= n_w) break;
-        const int c = a.queue[b_w + item];
-        const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
-        dedup_ctx<false>(s, a, c, region, pow2_at_least(2 * T), nullptr);
+    {
+        const int q = warp / 4;
+        const int n = a.counters[CNT_COUNT + CLS_DD_QUAD];
+        const int b = a.counters[CNT_BEGIN + CLS_DD_QUAD];
+        uint32_t* region = smem + q * 4 * DD_WARP_REGION;
+        for (;;) {
+            dd_sync<4>();
+            if ((warp & 3) == 0 && lane == 0) s_item[q] = atomicAdd(a.counters + CNT_HEAD + CLS_DD_QUAD, 1);
+            dd_sync<4>();
+            const int item = s_item[q];
+            if (item >= n) break;
+            const int c = a.queue[b + item];
+            const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
+            int E = pow2_at_least(2 * T);
+            if (E > DD_QUAD_E) E = DD_QUAD_E;
+#define F2_DD_QUAD(W) dedup_ctx<4, W>(s, a, c, region, E, wcnt + q * 4 * DD_K)
+            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_QUAD)
+#undef F2_DD_QUAD
+        }
+    }
+    {
+        const int n = a.counters[CNT_COUNT + CLS_DD_WARP];
+        const int b = a.counters[CNT_BEGIN + CLS_DD_WARP];
+        uint32_t* region = smem + warp * DD_WARP_REGION;
+        for (;;) {
+            int item = 0;
+            if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_WARP, 1);
+            item = __shfl_sync(FULL, item, 0);
+            if (item >= n) break;
+            const int c = a.queue[b + item];
+            const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
+            const int E = pow2_at_least(2 * T);
+#define F2_DD_WARP(W) dedup_ctx<1, W>(s, a, c, region, E, nullptr)
+            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_WARP)
+#undef F2_DD_WARP
+        }
     }
 }
 
@@ -617,9 +739,11 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     const long long seen = s.rows_seen[c];
     const int64_t r0 = a.row_off[c];
     const int64_t T = a.row_off[c + 1] - r0;
-    const int R = a.rep_count ? a.rep_count[c] : (int)T;
-    const int32_t* reps = a.rep_list ? a.rep_list + r0 : nullptr;
-    const int32_t* dups = a.rep_dup ? a.rep_dup + r0 : nullptr;
+    const int rc = a.rep_count ? a.rep_count[c] : -((int)T + 2);
+    const bool deduped = rc >= 0;
+    const int R = deduped ? rc : -(rc + 2);
+    const int32_t* reps = deduped ? a.rep_list + r0 : nullptr;
+    const int32_t* dups = deduped ? a.rep_dup + r0 : nullptr;
     const uint32_t* xc = a.x + a.x_off[c];
     const uint4* yc = a.y + r0;
     long long first = LLONG_MAX;
@@ -713,20 +837,6 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     group_sync<CTA>();
 }
 
-#define F2_NARROW_SWITCH(wd, CALL)   \
-    switch (wd) {                    \
-    case 1: CALL(1); break;          \
-    case 2: CALL(2); break;          \
-    case 3: CALL(3); break;          \
-    case 4: CALL(4); break;          \
-    case 5: CALL(5); break;          \
-    case 6: CALL(6); break;          \
-    case 7: CALL(7); break;          \
-    case 8: CALL(8); break;          \
-    case 9: CALL(9); break;          \
-    default: break;                  \
-    }
-
 __global__ void __launch_bounds__(LEARN_WARPS * 32, 2) elim_narrow_kernel(StoreDev s, LearnArgs a)
 {
     extern __shared__ __align__(16) uint32_t smem[];
@@ -780,81 +890,166 @@ __global__ void __launch_bounds__(WIDE_WARPS * 32) elim_wide_kernel(StoreDev s, 
     }
 }
 
-// Validate the batch and order the work longest-first (one block).
-//   mode 0 (dedup plan): every valid non-empty context goes to the warp or
-//     CTA dedup queue by its row count; rep_count[c] is set to -1 for an
-//     invalid context and 0 for an empty one (the dedup pass fills the rest);
-//   mode 1 (elimination plan): contexts with representatives (rep_count, or
-//     all rows when rep_count is NULL, after the same validation) go to the
+// Validate the batch and order the work longest-first, in three kernels:
+// per-context keys and a histogram (grid), the bucket offsets (one block),
+// and the scatter into the queue (grid).  A key is (class, work bucket,
+// width); within a class, buckets run from the most work to the least and,
+// inside a bucket, widths in increasing order (so few template variants run
+// at once).
+//   mode 0 (dedup plan): every valid non-empty context with at most DD_XW
+//     feature words goes to the warp, quad or CTA dedup queue by its row
+//     count; rep_count[c] becomes 0 (filled by the dedup pass), -1 (invalid,
+//     skipped) or -(T+2) (every row is its own representative);
+//   mode 1 (elimination plan): contexts with rows to eliminate go to the
 //     warp, CTA or wide elimination queue.
-__global__ void __launch_bounds__(1024) plan_kernel(StoreDev s, const int64_t* __restrict__ row_off,
-                                                    const int64_t* __restrict__ x_off, int64_t total_rows,
-                                                    int64_t total_xw, int32_t* __restrict__ rep_count, int mode,
-                                                    int warp_region_words, int64_t heavy_rows, int64_t warp_work,
-                                                    int32_t* __restrict__ queue, int32_t* __restrict__ keybuf,
-                                                    int* __restrict__ counters)
+constexpr int PLAN_SUB = PLAN_BUCKETS * NARROW_WD;  // (bucket, width) keys per class
+constexpr int PLAN_KEYS = NUM_CLASSES * PLAN_SUB;
+
+struct PlanArgs {
+    const int64_t* row_off;
+    const int64_t* x_off;
+    int64_t total_rows;
+    int64_t total_xw;
+    int32_t* rep_count;
+    int mode;
+    int warp_region_words;
+    int64_t heavy_rows;
+    int64_t warp_work;
+    int32_t* queue;
+    int32_t* keybuf;
+    int* hist;     // PLAN_KEYS counts (zeroed before plan_key_kernel), then cursors
+    int* counters;
+};
+
+__global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
 {
-    __shared__ int hist[NUM_CLASSES][PLAN_BUCKETS];
-    __shared__ int cursor[NUM_CLASSES][PLAN_BUCKETS];
-    for (int i = threadIdx.x; i < NUM_CLASSES * PLAN_BUCKETS; i += blockDim.x) (&hist[0][0])[i] = 0;
+    __shared__ int hist[PLAN_KEYS];
+    for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
         const CtxDesc cd = s.desc[c];
         int64_t R;
-        if (mode == 1 && rep_count) {
-            R = rep_count[c];
+        if (p.mode == 1 && p.rep_count) {
+            R = p.rep_count[c];
+            if (R <= -2) R = -(R + 2);
         } else {
-            const int64_t a0 = row_off[c], a1 = row_off[c + 1];
+            const int64_t a0 = p.row_off[c], a1 = p.row_off[c + 1];
             const int64_t rows = a1 - a0;
-            const int64_t x0 = x_off[c];
-            const bool ok = a0 >= 0 && rows >= 0 && rows < (1ll << 31) && a1 <= total_rows && x0 >= 0 &&
-                            rows <= total_xw && x0 + rows * cd.xw <= total_xw;
+            const int64_t x0 = p.x_off[c];
+            const bool ok = a0 >= 0 && rows >= 0 && rows < (1ll << 31) && a1 <= p.total_rows && x0 >= 0 &&
+                            rows <= p.total_xw && x0 + rows * cd.xw <= p.total_xw;
             if (!ok) record_status(s.status, F2_ERR_ROWS);
             R = ok ? rows : -1;
-            if (mode == 0 && rep_count) rep_count[c] = (R > 0) ? 0 : (int32_t)R;
+            if (p.mode == 0 && p.rep_count) {
+                if (R > 0 && cd.xw > DD_XW) {
+                    p.rep_count[c] = (int32_t)(-(R + 2));
+                    R = 0;
+                } else {
+                    p.rep_count[c] = (R > 0) ? 0 : (int32_t)R;
+                }
+            }
         }
         int key = -1;
         if (R > 0) {
             int cls;
             unsigned long long work;
-            if (mode == 0) {
-                cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : CLS_DD_CTA;
+            if (p.mode == 0) {
+                cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : (R <= DD_QUAD_MAX_ROWS ? CLS_DD_QUAD : CLS_DD_CTA);
                 work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
             } else {
                 if (cd.wd > NARROW_WD) cls = CLS_WIDE;
-                else if (elim_words(cd.d, cd.wd) > warp_region_words || R >= heavy_rows || R * cd.d > warp_work)
+                else if (elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
+                         R * cd.d > p.warp_work)
                     cls = CLS_CTA;
                 else cls = CLS_WARP;
                 work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
             }
             int bucket = 63 - __clzll(work);
             if (bucket >= PLAN_BUCKETS) bucket = PLAN_BUCKETS - 1;
-            key = cls * PLAN_BUCKETS + bucket;
-            atomicAdd(&hist[cls][bucket], 1);
+            const int width = (p.mode == 0 ? cd.xw : cd.wd);
+            const int sub = (PLAN_BUCKETS - 1 - bucket) * NARROW_WD + (width > NARROW_WD ? NARROW_WD : width) - 1;
+            key = cls * PLAN_SUB + sub;
+            atomicAdd(&hist[key], 1);
         }
-        keybuf[c] = key;
+        p.keybuf[c] = key;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        int pos = 0;
-        for (int cls = 0; cls < NUM_CLASSES; ++cls) {
-            counters[CNT_BEGIN + cls] = pos;
-            for (int bk = PLAN_BUCKETS - 1; bk >= 0; --bk) {
-                cursor[cls][bk] = pos;
-                pos += hist[cls][bk];
+    for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x)
+        if (hist[i]) atomicAdd(p.hist + i, hist[i]);
+}
+
+// Exclusive scan of the key counts in key order (one block of 1024).
+__global__ void __launch_bounds__(1024) plan_scan_kernel(PlanArgs p)
+{
+    constexpr int PER = (PLAN_KEYS + 1023) / 1024;
+    __shared__ int wsum[32];
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    int v[PER];
+    int tot = 0;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const int k = t * PER + j;
+        v[j] = (k < PLAN_KEYS) ? p.hist[k] : 0;
+        tot += v[j];
+    }
+    int inc = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(FULL, inc, o);
+        if (lane >= o) inc += u;
+    }
+    if (lane == 31) wsum[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        int w = wsum[lane];
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(FULL, wi, o);
+            if (lane >= o) wi += u;
+        }
+        wsum[lane] = wi - w;
+    }
+    __syncthreads();
+    int run = wsum[warp] + inc - tot;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const int k = t * PER + j;
+        if (k < PLAN_KEYS) {
+            p.hist[k] = run;  // becomes the cursor of key k
+            if (k % PLAN_SUB == 0) {
+                const int cls = k / PLAN_SUB;
+                p.counters[CNT_BEGIN + cls] = run;
+                p.counters[CNT_HEAD + cls] = 0;
             }
-            counters[CNT_COUNT + cls] = pos - counters[CNT_BEGIN + cls];
-            counters[CNT_HEAD + cls] = 0;
+            run += v[j];
+            if (k % PLAN_SUB == PLAN_SUB - 1) {
+                const int cls = k / PLAN_SUB;
+                p.counters[CNT_COUNT + cls] = run - p.counters[CNT_BEGIN + cls];
+            }
         }
     }
-    __syncthreads();
-    for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
-        const int key = keybuf[c];
-        if (key >= 0) {
-            const int p = atomicAdd(&cursor[key / PLAN_BUCKETS][key % PLAN_BUCKETS], 1);
-            queue[p] = c;
-        }
+}
+
+__global__ void __launch_bounds__(256) plan_scatter_kernel(StoreDev s, PlanArgs p)
+{
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
+        const int key = p.keybuf[c];
+        if (key >= 0) p.queue[atomicAdd(p.hist + key, 1)] = c;
     }
+}
+
+int launch_plan(const StoreDev& sd, const PlanArgs& pa, int num_sms, cudaStream_t cs)
+{
+    cudaError_t e = cudaMemsetAsync(pa.hist, 0, sizeof(int) * PLAN_KEYS, cs);
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    int blocks = (sd.num_ctx + 255) / 256;
+    if (blocks > num_sms * 2) blocks = num_sms * 2;
+    if (blocks < 1) blocks = 1;
+    plan_key_kernel<<<blocks, 256, 0, cs>>>(sd, pa);
+    plan_scan_kernel<<<1, 1024, 0, cs>>>(pa);
+    plan_scatter_kernel<<<blocks, 256, 0, cs>>>(sd, pa);
+    return f2_cuda_status(cudaGetLastError());
 }
 
 inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) == 0; }
@@ -870,13 +1065,26 @@ size_t narrow_smem(int max_narrow_words, int warp_region_words)
 // Enqueue pass 2 (plan + kernels) for one batch.
 int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* row_off, const int64_t* x_off,
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
-                       int64_t warp_work, int32_t* queue, int32_t* keybuf, int num_sms, int max_narrow_words,
-                       bool has_narrow, int max_wide_d, bool has_wide, cudaStream_t cs)
+                       int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
+                       int max_narrow_words, bool has_narrow, int max_wide_d, bool has_wide, cudaStream_t cs)
 {
-    plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off, x_off, total_rows, total_xw, rep_count, 1, la.warp_region_words,
-                                    heavy_rows, warp_work, queue, keybuf, la.counters);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return f2_cuda_status(e);
+    PlanArgs pa;
+    pa.row_off = row_off;
+    pa.x_off = x_off;
+    pa.total_rows = total_rows;
+    pa.total_xw = total_xw;
+    pa.rep_count = rep_count;
+    pa.mode = 1;
+    pa.warp_region_words = la.warp_region_words;
+    pa.heavy_rows = heavy_rows;
+    pa.warp_work = warp_work;
+    pa.queue = queue;
+    pa.keybuf = keybuf;
+    pa.hist = hist;
+    pa.counters = la.counters;
+    int rc = launch_plan(sd, pa, num_sms, cs);
+    if (rc != F2_OK) return rc;
+    cudaError_t e;
     if (has_narrow) {
         const size_t smem = narrow_smem(max_narrow_words, la.warp_region_words);
         e = cudaFuncSetAttribute(elim_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -947,10 +1155,22 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     const StoreDev sd = st->dev();
     if (dedup) {
-        plan_kernel<<<1, 1024, 0, cs>>>(sd, row_off, x_off, total_rows, total_x_words, st->rep_count, 0, 0, 0, 0,
-                                        st->queue, st->keybuf, st->counters);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        PlanArgs pa;
+        pa.row_off = row_off;
+        pa.x_off = x_off;
+        pa.total_rows = total_rows;
+        pa.total_xw = total_x_words;
+        pa.rep_count = st->rep_count;
+        pa.mode = 0;
+        pa.warp_region_words = 0;
+        pa.heavy_rows = 0;
+        pa.warp_work = 0;
+        pa.queue = st->queue;
+        pa.keybuf = st->keybuf;
+        pa.hist = st->plan_hist;
+        pa.counters = st->counters;
+        int rc = launch_plan(sd, pa, st->num_sms, cs);
+        if (rc != F2_OK) return rc;
         DedupArgs da;
         da.row_off = row_off;
         da.x_off = x_off;
@@ -983,8 +1203,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0, &max_narrow_words,
                   &has_narrow, &max_wide_d, &has_wide);
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
-                              st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->num_sms, max_narrow_words,
-                              has_narrow, max_wide_d, has_wide, cs);
+                              st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
+                              max_narrow_words, has_narrow, max_wide_d, has_wide, cs);
 }
 
 // ---------------------------------------------------------------------------
@@ -1002,6 +1222,7 @@ struct NoallocScratch {
     int32_t queue[F2_NOALLOC_MAX_CTX];
     int32_t keybuf[F2_NOALLOC_MAX_CTX];
     int counters[32];
+    int plan_hist[PLAN_KEYS];
 };
 
 // Device storage for the scratch; in host code this name is only a symbol
@@ -1185,6 +1406,6 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     bool has_narrow, has_wide;
     width_summary(n_bits_host, num_ctx, raw, &max_narrow_words, &has_narrow, &max_wide_d, &has_wide);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,
-                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, nd->num_sms, max_narrow_words, has_narrow,
-                              max_wide_d, has_wide, cs);
+                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, sc->plan_hist, nd->num_sms, max_narrow_words,
+                              has_narrow, max_wide_d, has_wide, cs);
 }
