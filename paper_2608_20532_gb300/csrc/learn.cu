@@ -318,57 +318,70 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
             for (int v = 0; v < XW; ++v) hh = fnv_step(hh, xv[j][v]);
             h[j] = fmix32(fnv_step(fnv_step(fnv_step(fnv_step(hh, yv[j].x), yv[j].y), yv[j].z), yv[j].w));
         }
-        // home slots (shared memory)
+        // probe by fingerprint only (shared memory): the first slot holding
+        // this fingerprint, or an empty slot that the row then claims
         uint2 ent[DD_K];
+        uint32_t cs[DD_K];
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
             const int i = base + j * NT + t;
             mine[j] = (i < T) ? -2 : -1;  // -2 = unresolved
             ent[j] = make_uint2(0u, 0u);
+            cs[j] = 0u;
             if (i < T) {
-                const uint32_t slot = (h[j] >> 7) & emask;
-                ent[j] = tab[slot];
-                if (ent[j].x == 0u) {
-                    const unsigned long long want = ((unsigned long long)(uint32_t)i << 32) | (h[j] | 1u);
-                    const unsigned long long old =
-                        atomicCAS(reinterpret_cast<unsigned long long*>(tab + slot), 0ull, want);
-                    if (old == 0ull) {
-                        mine[j] = (int)slot;
-                    } else {
-                        ent[j].x = (uint32_t)old;
-                        ent[j].y = (uint32_t)(old >> 32);
+                const uint32_t fp = h[j] | 1u;
+                uint32_t slot = (h[j] >> 7) & emask;
+                int p = 0;
+                for (; p < DEDUP_PROBES; ++p, slot = (slot + 1) & emask) {
+                    uint2 e = tab[slot];
+                    if (e.x == 0u) {
+                        const unsigned long long want = ((unsigned long long)(uint32_t)i << 32) | fp;
+                        const unsigned long long old =
+                            atomicCAS(reinterpret_cast<unsigned long long*>(tab + slot), 0ull, want);
+                        if (old == 0ull) {
+                            mine[j] = (int)slot;
+                            break;
+                        }
+                        e.x = (uint32_t)old;
+                        e.y = (uint32_t)(old >> 32);
+                    }
+                    if (e.x == fp) {
+                        ent[j] = e;
+                        cs[j] = slot;
+                        break;
                     }
                 }
+                if (p == DEDUP_PROBES) mine[j] = -1;  // table region full: own representative
             }
         }
-        // full comparison with the matching rows (loads issued together)
-        bool eq[DD_K];
+        // full comparison with the fingerprint matches: every load first
+        bool need[DD_K];
+        uint4 yo[DD_K];
+        uint32_t xo[DD_K][XW];
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
-            eq[j] = false;
-            if (mine[j] == -2 && ent[j].x == (h[j] | 1u)) {
-                const int64_t o = ent[j].y;
-                const uint4 yo = __ldg(yc + o);
-                bool e = yo.x == yv[j].x && yo.y == yv[j].y && yo.z == yv[j].z && yo.w == yv[j].w;
+            need[j] = mine[j] == -2;
+            const int64_t o = need[j] ? (int64_t)ent[j].y : 0;
+            yo[j] = need[j] ? __ldg(yc + o) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-                for (int v = 0; v < XW; ++v) {
-                    uint32_t w = __ldg(xc + o * XW + v);
-                    if (v == XW - 1) w &= lm;
-                    e = e && (w == xv[j][v]);
-                }
-                eq[j] = e;
-            }
+            for (int v = 0; v < XW; ++v) xo[j][v] = need[j] ? __ldg(xc + o * XW + v) : 0u;
         }
 #pragma unroll
         for (int j = 0; j < DD_K; ++j) {
-            if (mine[j] != -2) continue;
+            if (!need[j]) continue;
+            bool e = yo[j].x == yv[j].x && yo[j].y == yv[j].y && yo[j].z == yv[j].z && yo[j].w == yv[j].w;
+#pragma unroll
+            for (int v = 0; v < XW; ++v) {
+                const uint32_t w = (v == XW - 1) ? (xo[j][v] & lm) : xo[j][v];
+                e = e && (w == xv[j][v]);
+            }
             const int i = base + j * NT + t;
-            const uint32_t slot = (h[j] >> 7) & emask;
-            if (eq[j]) {
-                if ((uint32_t)i < ent[j].y) atomicMin(&tab[slot].y, (uint32_t)i);
-                mine[j] = (int)slot;
-            } else {  // slow path: keep probing
-                mine[j] = dd_find_insert(tab, E, h[j], i, yv[j], xc, yc, xw, n, (slot + 1) & emask, DEDUP_PROBES - 1);
+            if (e) {
+                if ((uint32_t)i < ent[j].y) atomicMin(&tab[cs[j]].y, (uint32_t)i);
+                mine[j] = (int)cs[j];
+            } else {  // a different row with the same fingerprint: keep probing
+                mine[j] = dd_find_insert(tab, E, h[j], i, yv[j], xc, yc, XW, n, (cs[j] + 1) & emask,
+                                         DEDUP_PROBES - 1);
             }
         }
         dd_sync<G>();
