@@ -293,26 +293,40 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
     }
     dd_sync<G>();
     int nrep = 0;
-    for (int base = 0; base < T; base += NT * DD_K) {
-        int mine[DD_K];
-        uint32_t h[DD_K];
-        uint4 yv[DD_K];
-        uint32_t xv[DD_K][XW];
-        // every load of the round first
+    // rows of the round in flight, and the next round's rows prefetched while
+    // the current one is probed and verified
+    constexpr int K = (XW <= 2) ? DD_K : 2;
+    uint4 yn[K];
+    uint32_t xn[K][XW];
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
-            const int i = base + j * NT + t;
-            const bool ok = i < T;
-            yv[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
+    for (int j = 0; j < K; ++j) {
+        const int i = j * NT + t;
+        const bool ok = i < T;
+        yn[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-            for (int v = 0; v < XW; ++v) {
-                uint32_t w = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
-                if (v == XW - 1) w &= lm;
-                xv[j][v] = w;
-            }
+        for (int v = 0; v < XW; ++v) xn[j][v] = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
+    }
+    for (int base = 0; base < T; base += NT * K) {
+        int mine[K];
+        uint32_t h[K];
+        uint4 yv[K];
+        uint32_t xv[K][XW];
+#pragma unroll
+        for (int j = 0; j < K; ++j) {
+            yv[j] = yn[j];
+#pragma unroll
+            for (int v = 0; v < XW; ++v) xv[j][v] = (v == XW - 1) ? (xn[j][v] & lm) : xn[j][v];
         }
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
+            const int i = base + NT * K + j * NT + t;
+            const bool ok = i < T;
+            yn[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int v = 0; v < XW; ++v) xn[j][v] = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < K; ++j) {
             uint32_t hh = 0x811C9DC5u;
 #pragma unroll
             for (int v = 0; v < XW; ++v) hh = fnv_step(hh, xv[j][v]);
@@ -320,10 +334,10 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
         }
         // probe by fingerprint only (shared memory): the first slot holding
         // this fingerprint, or an empty slot that the row then claims
-        uint2 ent[DD_K];
-        uint32_t cs[DD_K];
+        uint2 ent[K];
+        uint32_t cs[K];
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
             const int i = base + j * NT + t;
             mine[j] = (i < T) ? -2 : -1;  // -2 = unresolved
             ent[j] = make_uint2(0u, 0u);
@@ -355,11 +369,11 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
             }
         }
         // full comparison with the fingerprint matches: every load first
-        bool need[DD_K];
-        uint4 yo[DD_K];
-        uint32_t xo[DD_K][XW];
+        bool need[K];
+        uint4 yo[K];
+        uint32_t xo[K][XW];
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
             need[j] = mine[j] == -2;
             const int64_t o = need[j] ? (int64_t)ent[j].y : 0;
             yo[j] = need[j] ? __ldg(yc + o) : make_uint4(0, 0, 0, 0);
@@ -367,7 +381,7 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
             for (int v = 0; v < XW; ++v) xo[j][v] = need[j] ? __ldg(xc + o * XW + v) : 0u;
         }
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
             if (!need[j]) continue;
             bool e = yo[j].x == yv[j].x && yo[j].y == yv[j].y && yo[j].z == yv[j].z && yo[j].w == yv[j].w;
 #pragma unroll
@@ -385,25 +399,25 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
             }
         }
         dd_sync<G>();
-        uint32_t bal[DD_K];
+        uint32_t bal[K];
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
             const int i = base + j * NT + t;
             const bool valid = i < T;
             const int rep = (valid && mine[j] >= 0) ? (int)tab[mine[j]].y : i;
             const bool isrep = valid && rep == i;
             if (valid && !isrep) atomicAdd(D + mine[j], 1);
             bal[j] = __ballot_sync(FULL, isrep);
-            if (G > 1 && lane == 0) wcnt[gw * DD_K + j] = __popc(bal[j]);
+            if (G > 1 && lane == 0) wcnt[gw * K + j] = __popc(bal[j]);
         }
         if (G > 1) dd_sync<G>();
 #pragma unroll
-        for (int j = 0; j < DD_K; ++j) {
+        for (int j = 0; j < K; ++j) {
             int before = 0, total = __popc(bal[j]);
             if (G > 1) {
                 total = 0;
                 for (int ww = 0; ww < G; ++ww) {
-                    const int v = wcnt[ww * DD_K + j];
+                    const int v = wcnt[ww * K + j];
                     if (ww < gw) before += v;
                     total += v;
                 }
