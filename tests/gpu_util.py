@@ -92,3 +92,40 @@ def csr_from_rows(n_bits, rows_per_ctx):
             x[x_off[c] + i * W[c]: x_off[c] + (i + 1) * W[c]] = xw
             y[row_off[c] + i] = yw
     return row_off, x_off, x, y
+
+
+def oracle_for_contexts(wl, ctxs, threads=None):
+    """Oracle over the rows of the chosen contexts only (all batches, stream
+    order), learned in parallel.  Returns (oracle, export); context ctxs[j]
+    is the oracle's context j."""
+    ctxs = np.asarray(ctxs)
+    xs, ys, rows = [], [], []
+    for c in ctxs:
+        x, y = wl.ctx_rows(int(c))
+        xs.append(np.ascontiguousarray(x).reshape(-1))
+        ys.append(np.ascontiguousarray(y))
+        rows.append(len(y))
+    nb = wl.n_bits[ctxs]
+    W = (nb.astype(np.int64) + 31) // 32
+    cnt = np.array(rows, np.int64)
+    row_off = np.zeros(len(ctxs) + 1, np.int64)
+    row_off[1:] = np.cumsum(cnt)
+    x_off = np.concatenate([[0], np.cumsum(cnt * W)[:-1]]).astype(np.int64)
+    O = oracle.Oracle(nb, threads=threads or len(ctxs))
+    O.learn(row_off, x_off, np.concatenate(xs), np.concatenate(ys))
+    return O, O.export()
+
+
+def assert_contexts_equal(binding, got, store, ref, ref_layout, ctxs):
+    """Context ctxs[j] of the GPU store equals context j of the oracle."""
+    g = {k: binding.to_numpy(got[k]) for k in KEYS}
+    for j, c in enumerate(np.asarray(ctxs)):
+        c = int(c)
+        for k in ("rank", "contra", "first_contra", "n_contra", "rows_seen"):
+            assert as_bytes(g[k][c:c + 1]).tobytes() == as_bytes(ref[k][j:j + 1]).tobytes(), (k, c)
+        pairs = (("pivot_mask", store.pw_off, "pw_off"), ("basis_x", store.xw_off, "xw_off"),
+                 ("basis_z", store.slot_off, "slot_off"))
+        for k, off, lk in pairs:
+            a = g[k][int(off[c]):int(off[c + 1])]
+            b = ref[k][int(ref_layout[lk][j]):int(ref_layout[lk][j + 1])]
+            assert np.array_equal(as_bytes(a), as_bytes(b)), (k, c)
