@@ -406,14 +406,14 @@ def run_ours(args):
     t_hbm, t_alu = bytes_learn / hbm_peak, ops_learn / alu_peak
     learn_bound = "hbm" if t_hbm >= t_alu else "alu"
     rl_learn = {
-        "kernel": "f2_learn_batched (plan_kernel + learn_narrow_kernel)",
+        "kernel": "f2_learn_batched (plan kernels + dedup_kernel + elim_narrow_kernel)",
         "hbm": {"achieved": bytes_learn / learn_mean / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": (bytes_learn / learn_mean) / hbm_peak, "bytes_per_launch": bytes_learn},
         "alu": {"achieved": ops_learn / learn_mean / 1e12, "peak": alu_peak / 1e12, "unit": "Tops/s",
                 "frac": (ops_learn / learn_mean) / alu_peak, "ops_per_launch": ops_learn,
                 "peak_probe_lop3": (probe / 1e12) if probe else None},
     }
-    traffic = profile_traffic("learn_narrow_kernel")
+    traffic = profile_traffic("f2_learn_batched")
     dom = rl_learn[learn_bound]
     roofline = {"bound": learn_bound, "achieved": dom["achieved"], "peak": dom["peak"], "unit": dom["unit"],
                 "frac": dom["frac"], "traffic": traffic,
