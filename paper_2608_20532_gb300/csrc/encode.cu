@@ -85,34 +85,88 @@ __device__ __forceinline__ bool encode_one(const StoreDev& s, const CtxDesc& cd,
     return resid == 0;
 }
 
-__global__ void __launch_bounds__(256, 3) encode_kernel(StoreDev s, int64_t Q, const int32_t* __restrict__ ctx_id,
-                                                     const uint32_t* __restrict__ x, int stride,
-                                                     uint4* __restrict__ y, uint8_t* __restrict__ in_span)
+constexpr int ENC_THREADS = 256;
+constexpr int ENC_CHUNK = 2048;    // queries grouped per CTA step
+constexpr int ENC_BUCKETS = 256;   // context-hash buckets of a chunk
+
+__device__ __forceinline__ void encode_query(const StoreDev& s, int64_t i, const int32_t* __restrict__ ctx_id,
+                                             const uint32_t* __restrict__ x, int stride, uint4* __restrict__ y,
+                                             uint8_t* __restrict__ in_span)
 {
-    const int64_t step = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < Q; i += step) {
-        const int c = __ldg(ctx_id + i);
-        uint4 acc = make_uint4(0, 0, 0, 0);
-        uint8_t flag;
-        if (c < 0 || c >= s.num_ctx) {
-            record_status(s.status, F2_ERR_CTX_RANGE);
+    const int c = __ldg(ctx_id + i);
+    uint4 acc = make_uint4(0, 0, 0, 0);
+    uint8_t flag;
+    if (c < 0 || c >= s.num_ctx) {
+        record_status(s.status, F2_ERR_CTX_RANGE);
+        flag = 0xFF;
+    } else {
+        const CtxDesc cd = s.desc[c];
+        const uint32_t* xq = x + i * stride;
+        bool ok;
+        if (cd.xw > stride) {
+            record_status(s.status, F2_ERR_STRIDE);
             flag = 0xFF;
+            ok = false;
         } else {
-            const CtxDesc cd = s.desc[c];
-            const uint32_t* xq = x + i * stride;
-            bool ok;
-            if (cd.xw > stride) {
-                record_status(s.status, F2_ERR_STRIDE);
-                flag = 0xFF;
-                ok = false;
-            } else {
-                ok = (cd.wd <= NARROW_WD) ? encode_one<NARROW_WD>(s, cd, xq, acc) : encode_one<33>(s, cd, xq, acc);
-                flag = ok ? 1 : 0;
-            }
-            if (!ok) acc = make_uint4(0, 0, 0, 0);
+            ok = (cd.wd <= NARROW_WD) ? encode_one<NARROW_WD>(s, cd, xq, acc) : encode_one<33>(s, cd, xq, acc);
+            flag = ok ? 1 : 0;
         }
-        y[i] = acc;
-        in_span[i] = flag;
+        if (!ok) acc = make_uint4(0, 0, 0, 0);
+    }
+    y[i] = acc;
+    in_span[i] = flag;
+}
+
+// Each CTA step takes ENC_CHUNK consecutive queries, partitions them in
+// shared memory by a hash of their context id (a counting sort into
+// ENC_BUCKETS buckets), and lets every thread encode the queries of the
+// permuted order: a warp then mostly serves queries of one context, which
+// share its basis rows in L1 and take similar paths.
+__global__ void __launch_bounds__(ENC_THREADS, 3) encode_kernel(StoreDev s, int64_t Q, const int32_t* __restrict__ ctx_id,
+                                                                const uint32_t* __restrict__ x, int stride,
+                                                                uint4* __restrict__ y, uint8_t* __restrict__ in_span)
+{
+    __shared__ int hist[ENC_BUCKETS];
+    __shared__ uint16_t perm[ENC_CHUNK];
+    __shared__ uint8_t key[ENC_CHUNK];
+    const int t = threadIdx.x;
+    for (int64_t base = (int64_t)blockIdx.x * ENC_CHUNK; base < Q; base += (int64_t)gridDim.x * ENC_CHUNK) {
+        const int n = (int)((Q - base) < ENC_CHUNK ? (Q - base) : ENC_CHUNK);
+        hist[t] = 0;
+        __syncthreads();
+        for (int k = t; k < n; k += ENC_THREADS) {
+            const uint32_t c = (uint32_t)__ldg(ctx_id + base + k);
+            const uint8_t b = (uint8_t)((c * 2654435761u) >> 24);
+            key[k] = b;
+            atomicAdd(&hist[b], 1);
+        }
+        __syncthreads();
+        if (t < 32) {  // exclusive scan of 256 bucket counts by one warp
+            int v[ENC_BUCKETS / 32];
+            int sum = 0;
+#pragma unroll
+            for (int j = 0; j < ENC_BUCKETS / 32; ++j) {
+                v[j] = hist[t * (ENC_BUCKETS / 32) + j];
+                sum += v[j];
+            }
+            int inc = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(FULL, inc, o);
+                if (t >= o) inc += u;
+            }
+            int run = inc - sum;
+#pragma unroll
+            for (int j = 0; j < ENC_BUCKETS / 32; ++j) {
+                hist[t * (ENC_BUCKETS / 32) + j] = run;
+                run += v[j];
+            }
+        }
+        __syncthreads();
+        for (int k = t; k < n; k += ENC_THREADS) perm[atomicAdd(&hist[key[k]], 1)] = (uint16_t)k;
+        __syncthreads();
+        for (int k = t; k < n; k += ENC_THREADS) encode_query(s, base + perm[k], ctx_id, x, stride, y, in_span);
+        __syncthreads();
     }
 }
 
@@ -126,10 +180,10 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
     if (!ctx_id || !x || !y_out || !in_span) return F2_ERR_INVALID_ARG;
     if (((uintptr_t)y_out % 16) != 0 || ((uintptr_t)x % 4) != 0 || ((uintptr_t)ctx_id % 4) != 0)
         return F2_ERR_ALIGN;
-    int64_t blocks = (Q + 255) / 256;
-    const int64_t cap = (int64_t)st->num_sms * 8;
+    int64_t blocks = (Q + ENC_CHUNK - 1) / ENC_CHUNK;
+    const int64_t cap = (int64_t)st->num_sms * 3;
     if (blocks > cap) blocks = cap;
-    encode_kernel<<<(int)blocks, 256, 0, (cudaStream_t)stream>>>(st->dev(), Q, ctx_id, x, x_stride_words,
-                                                                 reinterpret_cast<uint4*>(y_out), in_span);
+    encode_kernel<<<(int)blocks, ENC_THREADS, 0, (cudaStream_t)stream>>>(
+        st->dev(), Q, ctx_id, x, x_stride_words, reinterpret_cast<uint4*>(y_out), in_span);
     return f2_cuda_status(cudaGetLastError());
 }
