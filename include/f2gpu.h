@@ -166,8 +166,11 @@ int f2_solve_affine(const f2_store* store, uint32_t* W_dev, f2_stream_t stream);
  * and zero otherwise; in_span_dev[q] receives 1 (supported), 0 (rejected) or
  * 0xFF (context id out of range -- F2_ERR_CTX_RANGE is recorded -- or the
  * context needs more than x_stride_words words -- F2_ERR_STRIDE).
+ * The queries are grouped by context on the device first; the store keeps
+ * that scratch (20 bytes per query, at most 2^25 queries per pass, plus 4
+ * bytes per context) and grows it stream-ordered with cudaMallocAsync.
  * Errors: F2_ERR_INVALID_ARG (Q < 0, NULL pointers, x_stride_words < 1),
- * F2_ERR_ALIGN (y_out_dev not 16-byte aligned).
+ * F2_ERR_ALIGN (y_out_dev not 16-byte aligned), F2_ERR_OOM (scratch).
  */
 int f2_encode_batched(const f2_store* store, int64_t Q, const int32_t* ctx_id_dev,
                       const uint32_t* x_dev, int32_t x_stride_words, uint32_t* y_out_dev,
@@ -196,8 +199,11 @@ enum f2_option {
     F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA */
     F2_OPT_WARP_BASIS_BYTES = 2, /* shared memory (bytes) of one warp-owned context */
     F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context */
-    F2_OPT_DEDUP = 4             /* 1 (default): eliminate only the first occurrence of each distinct
+    F2_OPT_DEDUP = 4,            /* 1 (default): eliminate only the first occurrence of each distinct
                                     row and classify its repeats with it; 0: eliminate every row */
+    F2_OPT_ENCODE_TABLE_MIN = 5  /* shortest run of queries of one context (within a block of 2,048
+                                    grouped queries) encoded with a lookup table of its basis; default
+                                    32, at least 16; a value above 2,048 disables the tables */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -32,6 +32,7 @@ F2_OPT_HEAVY_ROWS = 1
 F2_OPT_WARP_BASIS_BYTES = 2
 F2_OPT_WARP_WORK = 3
 F2_OPT_DEDUP = 4
+F2_OPT_ENCODE_TABLE_MIN = 5
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

@@ -116,6 +116,15 @@ struct f2_store {
     int32_t* rep_list;      // per-row scratch of pass 1 (capacity rep_capacity rows)
     int32_t* rep_dup;
     int64_t rep_capacity;
+    // scratch of f2_encode_batched (grouping of the queries by context)
+    mutable int32_t* enc_bins;              // bucket sizes / starts, tile sums, ticket
+    mutable int64_t enc_bin_cap;
+    mutable int32_t* enc_off;               // offset of each query inside its bucket
+    mutable unsigned long long* enc_sorted; // (bucket << 32) | query, grouped
+    mutable unsigned long long* enc_items;  // runs left to the per-warp kernel
+    mutable int64_t enc_q_cap;
+    mutable int enc_short_per_sm;           // resident CTAs of the per-warp encode kernel
+    int enc_table_min;                      // shortest run encoded with a table
 
     f2::StoreDev dev() const
     {
@@ -136,5 +145,7 @@ struct f2_store {
     }
 };
 
-// Host helpers (store.cu).
+// Host helpers (store.cu, encode.cu).
 int f2_cuda_status(cudaError_t e);
+int f2_encode_table_min_default();
+int f2_encode_table_min_floor();

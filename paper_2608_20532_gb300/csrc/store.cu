@@ -39,7 +39,8 @@ static void free_store(f2_store* s)
     if (!s) return;
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
-                    s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup};
+                    s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
+                    s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     delete s;
@@ -81,6 +82,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->warp_basis_bytes = DEFAULT_WARP_REGION_BYTES;
     s->warp_work = DEFAULT_WARP_WORK;
     s->dedup = 1;
+    s->enc_table_min = f2_encode_table_min_default();
     if (cudaGetDevice(&s->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
         delete s;
@@ -369,6 +371,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_DEDUP:
         if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
         s->dedup = (int)value;
+        return F2_OK;
+    case F2_OPT_ENCODE_TABLE_MIN:
+        if (value < f2_encode_table_min_floor() || value > (int64_t(1) << 30)) return F2_ERR_INVALID_ARG;
+        s->enc_table_min = (int)value;
         return F2_OK;
     default:
         return F2_ERR_INVALID_ARG;
