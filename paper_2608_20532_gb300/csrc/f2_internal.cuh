@@ -28,8 +28,9 @@ enum Counter {
     CNT_COUNT = 16, // + class: number of contexts of each class
     CNT_WORDS = 32
 };
-// Work classes: elimination by a CTA / the wide kernel / a warp, and dedup
-// by a CTA / a quad of warps / a warp.
+// Work classes: elimination by a CTA / the wide kernel / a warp, dedup by a
+// CTA / a quad of warps / a warp, and elimination of the small-width contexts
+// (wd <= SMALL_WD, their own kernel) by a CTA / a warp.
 enum Class {
     CLS_CTA = 0,
     CLS_WIDE = 1,
@@ -37,8 +38,12 @@ enum Class {
     CLS_DD_CTA = 3,
     CLS_DD_QUAD = 4,
     CLS_DD_WARP = 5,
-    NUM_CLASSES = 6
+    CLS_CTA_S = 6,
+    CLS_WARP_S = 7,
+    NUM_CLASSES = 8
 };
+static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
+constexpr int SMALL_WD = 3;  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {

@@ -100,6 +100,25 @@ static_assert(DD_WARPS * DD_WARP_REGION * 4 <= DD_SMEM, "warp regions exceed the
 __host__ __device__ __forceinline__ int elim_words(int d, int wd) { return CTL_WORDS + d * row_stride(wd); }
 
 // Dispatch on a width 1..9 (feature words) to a template instantiation.
+#define F2_SMALL_SWITCH(wd, CALL)    \
+    switch (wd) {                    \
+    case 1: CALL(1); break;          \
+    case 2: CALL(2); break;          \
+    case 3: CALL(3); break;          \
+    default: break;                  \
+    }
+
+#define F2_BIG_SWITCH(wd, CALL)      \
+    switch (wd) {                    \
+    case 4: CALL(4); break;          \
+    case 5: CALL(5); break;          \
+    case 6: CALL(6); break;          \
+    case 7: CALL(7); break;          \
+    case 8: CALL(8); break;          \
+    case 9: CALL(9); break;          \
+    default: break;                  \
+    }
+
 #define F2_NARROW_SWITCH(wd, CALL)   \
     switch (wd) {                    \
     case 1: CALL(1); break;          \
@@ -518,30 +537,42 @@ __device__ __forceinline__ void reduce_snapshot(uint32_t (&xr)[WD], uint4& yr, c
                                                 const uint32_t (&P)[WD], uint64_t mixed)
 {
     constexpr int RS = row_stride(WD);
+    // A stored row never changes another pivot bit of the lane's row, so the
+    // bit that selects row b is the row's own bit b however the rows are
+    // ordered: two pivots are taken per step, their loads issued together.
 #pragma unroll
     for (int w = 0; w < WD; ++w) {
         uint32_t uw = __reduce_or_sync(FULL, xr[w] & P[w]);
         const bool xwork = (mixed & ((2ull << w) - 1ull)) != 0;
+        const uint32_t sel = xr[w];
         while (uw) {
-            const int b = __ffs(uw) - 1;
+            const int b0 = __ffs(uw) - 1;
             uw &= uw - 1;
-            const uint32_t* row = S + (32 * w + b) * RS;
-            const uint32_t m = 0u - ((xr[w] >> b) & 1u);
-            const uint4 z = *reinterpret_cast<const uint4*>(row);
-            yr.x ^= z.x & m;
-            yr.y ^= z.y & m;
-            yr.z ^= z.z & m;
-            yr.w ^= z.w & m;
+            const bool two = uw != 0u;
+            const int b1 = two ? __ffs(uw) - 1 : b0;
+            uw &= uw - 1;
+            const uint32_t* row0 = S + (32 * w + b0) * RS;
+            const uint32_t* row1 = S + (32 * w + b1) * RS;
+            const uint32_t m0 = 0u - ((sel >> b0) & 1u);
+            const uint32_t m1 = two ? 0u - ((sel >> b1) & 1u) : 0u;
+            const uint4 z0 = *reinterpret_cast<const uint4*>(row0);
+            const uint4 z1 = *reinterpret_cast<const uint4*>(row1);
+            yr.x ^= (z0.x & m0) ^ (z1.x & m1);
+            yr.y ^= (z0.y & m0) ^ (z1.y & m1);
+            yr.z ^= (z0.z & m0) ^ (z1.z & m1);
+            yr.w ^= (z0.w & m0) ^ (z1.w & m1);
             if (xwork) {
 #pragma unroll
                 for (int v4 = 0; v4 <= w / 4; ++v4) {
-                    const uint4 xv = *reinterpret_cast<const uint4*>(row + 4 + 4 * v4);
-                    const uint32_t e[4] = {xv.x, xv.y, xv.z, xv.w};
+                    const uint4 xa = *reinterpret_cast<const uint4*>(row0 + 4 + 4 * v4);
+                    const uint4 xb = *reinterpret_cast<const uint4*>(row1 + 4 + 4 * v4);
+                    const uint32_t ea[4] = {xa.x, xa.y, xa.z, xa.w};
+                    const uint32_t eb[4] = {xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const int v = 4 * v4 + j;
                         if (v <= w && v < WD)
-                            if ((mixed >> v) & 1ull) xr[v] ^= e[j] & m;
+                            if ((mixed >> v) & 1ull) xr[v] ^= (ea[j] & m0) ^ (eb[j] & m1);
                     }
                 }
             }
@@ -864,37 +895,56 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     group_sync<CTA>();
 }
 
-__global__ void __launch_bounds__(LEARN_WARPS * 32, 2) elim_narrow_kernel(StoreDev s, LearnArgs a)
+// Narrow elimination: CTA-owned contexts first (longest first), then
+// warp-owned ones.  SMALL: the contexts of at most SMALL_WD words, with
+// fixed 4 KB warp regions and a register budget for four CTAs per SM; else
+// the contexts of SMALL_WD + 1 .. NARROW_WD words.
+constexpr int SMALL_REGION_WORDS = 1024;
+static_assert(SMALL_REGION_WORDS >= 32 * SMALL_WD * row_stride(SMALL_WD) + CTL_WORDS,
+              "a warp region holds the basis of any small-width context");
+
+template <bool SMALL>
+__global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_kernel(StoreDev s, LearnArgs a)
 {
+    constexpr int C_CTA = SMALL ? CLS_CTA_S : CLS_CTA;
+    constexpr int C_WARP = SMALL ? CLS_WARP_S : CLS_WARP;
     extern __shared__ __align__(16) uint32_t smem[];
     __shared__ int s_item;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_cta = a.counters[CNT_COUNT + CLS_CTA];
-    const int b_cta = a.counters[CNT_BEGIN + CLS_CTA];
+    const int n_cta = a.counters[CNT_COUNT + C_CTA];
+    const int b_cta = a.counters[CNT_BEGIN + C_CTA];
     for (;;) {
         __syncthreads();
-        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_CTA, 1);
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + C_CTA, 1);
         __syncthreads();
         const int item = s_item;
         if (item >= n_cta) break;
         const int c = a.queue[b_cta + item];
         const int wd = s.desc[c].wd;
 #define F2_CALL_CTA(W) elim_ctx<W, true>(s, a, c, smem)
-        F2_NARROW_SWITCH(wd, F2_CALL_CTA)
+        if (SMALL) {
+            F2_SMALL_SWITCH(wd, F2_CALL_CTA)
+        } else {
+            F2_BIG_SWITCH(wd, F2_CALL_CTA)
+        }
 #undef F2_CALL_CTA
     }
-    const int n_w = a.counters[CNT_COUNT + CLS_WARP];
-    const int b_w = a.counters[CNT_BEGIN + CLS_WARP];
-    uint32_t* region = smem + warp * a.warp_region_words;
+    const int n_w = a.counters[CNT_COUNT + C_WARP];
+    const int b_w = a.counters[CNT_BEGIN + C_WARP];
+    uint32_t* region = smem + warp * (SMALL ? SMALL_REGION_WORDS : a.warp_region_words);
     for (;;) {
         int item = 0;
-        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_WARP, 1);
+        if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + C_WARP, 1);
         item = __shfl_sync(FULL, item, 0);
         if (item >= n_w) break;
         const int c = a.queue[b_w + item];
         const int wd = s.desc[c].wd;
 #define F2_CALL_WARP(W) elim_ctx<W, false>(s, a, c, region)
-        F2_NARROW_SWITCH(wd, F2_CALL_WARP)
+        if (SMALL) {
+            F2_SMALL_SWITCH(wd, F2_CALL_WARP)
+        } else {
+            F2_BIG_SWITCH(wd, F2_CALL_WARP)
+        }
 #undef F2_CALL_WARP
     }
 }
@@ -984,11 +1034,11 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
                 cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : (R <= DD_QUAD_MAX_ROWS ? CLS_DD_QUAD : CLS_DD_CTA);
                 work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
             } else {
+                const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
+                                   R * cd.d > p.warp_work;
                 if (cd.wd > NARROW_WD) cls = CLS_WIDE;
-                else if (elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
-                         R * cd.d > p.warp_work)
-                    cls = CLS_CTA;
-                else cls = CLS_WARP;
+                else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
+                else cls = heavy ? CLS_CTA : CLS_WARP;
                 work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
             }
             int bucket = 63 - __clzll(work);
@@ -1082,6 +1132,12 @@ int launch_plan(const StoreDev& sd, const PlanArgs& pa, int num_sms, cudaStream_
 inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) == 0; }
 
 // Shared-memory need of the narrow elimination kernel for a set of widths.
+// Which elimination kernels a store needs, and their widest bases.
+struct Widths {
+    int max_small_words = 0, max_narrow_words = 0, max_wide_d = 0;
+    bool has_small = false, has_narrow = false, has_wide = false;
+};
+
 size_t narrow_smem(int max_narrow_words, int warp_region_words)
 {
     const size_t cta = 4 * (size_t)max_narrow_words;
@@ -1093,7 +1149,7 @@ size_t narrow_smem(int max_narrow_words, int warp_region_words)
 int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* row_off, const int64_t* x_off,
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
-                       int max_narrow_words, bool has_narrow, int max_wide_d, bool has_wide, cudaStream_t cs)
+                       const Widths& wv, cudaStream_t cs)
 {
     PlanArgs pa;
     pa.row_off = row_off;
@@ -1112,20 +1168,28 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     int rc = launch_plan(sd, pa, num_sms, cs);
     if (rc != F2_OK) return rc;
     cudaError_t e;
-    if (has_narrow) {
-        const size_t smem = narrow_smem(max_narrow_words, la.warp_region_words);
-        e = cudaFuncSetAttribute(elim_narrow_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+    auto narrow = [&](auto kernel, size_t smem) -> int {
+        cudaError_t er = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (er != cudaSuccess) return f2_cuda_status(er);
         int per_sm = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, elim_narrow_kernel, LEARN_WARPS * 32, smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, LEARN_WARPS * 32, smem);
+        if (er != cudaSuccess) return f2_cuda_status(er);
         if (per_sm < 1) per_sm = 1;
-        elim_narrow_kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
+        return f2_cuda_status(cudaGetLastError());
+    };
+    if (wv.has_small) {
+        const size_t words = (size_t)LEARN_WARPS * SMALL_REGION_WORDS;
+        rc = narrow(elim_narrow_kernel<true>,
+                    4 * (words > (size_t)wv.max_small_words ? words : (size_t)wv.max_small_words));
+        if (rc != F2_OK) return rc;
     }
-    if (has_wide) {
-        const size_t smem = 4 * (size_t)elim_words(max_wide_d, WIDE_WD);
+    if (wv.has_narrow) {
+        rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words));
+        if (rc != F2_OK) return rc;
+    }
+    if (wv.has_wide) {
+        const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
         e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return f2_cuda_status(e);
         elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, cs>>>(sd, la);
@@ -1135,25 +1199,25 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     return F2_OK;
 }
 
-// Widest narrow basis (words of an elimination group) and widest row.
-void width_summary(const int32_t* n_bits, int32_t num_ctx, bool raw, int* max_narrow_words, bool* has_narrow,
-                   int* max_wide_d, bool* has_wide)
+Widths width_summary(const int32_t* n_bits, int32_t num_ctx, bool raw)
 {
-    *max_narrow_words = 0;
-    *max_wide_d = 0;
-    *has_narrow = *has_wide = false;
+    Widths w;
     for (int32_t c = 0; c < num_ctx; ++c) {
         const int d = raw ? n_bits[c] : n_bits[c] + 1;
         const int wd = (d + 31) / 32;
-        if (wd <= NARROW_WD) {
-            *has_narrow = true;
-            const int w = elim_words(d, wd);
-            if (w > *max_narrow_words) *max_narrow_words = w;
+        const int words = elim_words(d, wd);
+        if (wd <= SMALL_WD) {
+            w.has_small = true;
+            if (words > w.max_small_words) w.max_small_words = words;
+        } else if (wd <= NARROW_WD) {
+            w.has_narrow = true;
+            if (words > w.max_narrow_words) w.max_narrow_words = words;
         } else {
-            *has_wide = true;
-            if (d > *max_wide_d) *max_wide_d = d;
+            w.has_wide = true;
+            if (d > w.max_wide_d) w.max_wide_d = d;
         }
     }
+    return w;
 }
 
 }  // namespace
@@ -1225,13 +1289,10 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     la.queue = st->queue;
     la.counters = st->counters;
     la.warp_region_words = (int)(st->warp_basis_bytes / 4);
-    int max_narrow_words, max_wide_d;
-    bool has_narrow, has_wide;
-    width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0, &max_narrow_words,
-                  &has_narrow, &max_wide_d, &has_wide);
+    const Widths wv = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
-                              max_narrow_words, has_narrow, max_wide_d, has_wide, cs);
+                              wv, cs);
 }
 
 // ---------------------------------------------------------------------------
@@ -1429,10 +1490,7 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     la.queue = sc->queue;
     la.counters = sc->counters;
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
-    int max_narrow_words, max_wide_d;
-    bool has_narrow, has_wide;
-    width_summary(n_bits_host, num_ctx, raw, &max_narrow_words, &has_narrow, &max_wide_d, &has_wide);
+    const Widths wv = width_summary(n_bits_host, num_ctx, raw);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,
-                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, sc->plan_hist, nd->num_sms, max_narrow_words,
-                              has_narrow, max_wide_d, has_wide, cs);
+                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, sc->plan_hist, nd->num_sms, wv, cs);
 }
