@@ -471,11 +471,12 @@ def run_ours(args):
 
 def launches_per_step(wl, has_q: bool) -> int:
     """Kernels one step enqueues (the host logic of the library): per learn
-    call a plan (3 kernels) and dedup_kernel for the duplicate pass, a plan and
+    call a plan (3 kernels) and dedup_kernel for the duplicate pass, a plan,
     the elimination kernel of each width class present (d <= 96, 96 < d <=
-    288, wider); solve_kernel; per 2^25 queries the five encode kernels."""
+    288, wider) and the full-rank check; solve_kernel; per 2^25 queries the
+    five encode kernels."""
     wd = (wl.n_bits.astype(np.int64) + 1 + 31) // 32
-    learn = 3 + 1 + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any()) + int(store_has_wide(wl))
+    learn = 3 + 1 + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any()) + int(store_has_wide(wl)) + 1
     enc = 5 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
     return len(wl.batches) * learn + 1 + enc
 

@@ -24,13 +24,14 @@ constexpr long long DEFAULT_WARP_WORK = 131072;   // largest rows x d handled by
 // Scheduling counters written by the plan kernel, read by the learn kernels.
 enum Counter {
     CNT_HEAD = 0,   // + class: next queue item of each class
-    CNT_BEGIN = 8,  // + class: first queue slot of each class
-    CNT_COUNT = 16, // + class: number of contexts of each class
-    CNT_WORDS = 32
+    CNT_BEGIN = 16, // + class: first queue slot of each class
+    CNT_COUNT = 32, // + class: number of contexts of each class
+    CNT_WORDS = 48
 };
 // Work classes: elimination by a CTA / the wide kernel / a warp, dedup by a
-// CTA / a quad of warps / a warp, and elimination of the small-width contexts
-// (wd <= SMALL_WD, their own kernel) by a CTA / a warp.
+// CTA / a quad of warps / a warp, elimination of the small-width contexts
+// (wd <= SMALL_WD, their own kernel) by a CTA / a warp, and the contexts of
+// full rank at the start of a call (rows checked independently).
 enum Class {
     CLS_CTA = 0,
     CLS_WIDE = 1,
@@ -40,10 +41,12 @@ enum Class {
     CLS_DD_WARP = 5,
     CLS_CTA_S = 6,
     CLS_WARP_S = 7,
-    NUM_CLASSES = 8
+    CLS_FULL = 8,
+    NUM_CLASSES = 9
 };
 static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
-constexpr int SMALL_WD = 3;  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
+constexpr int SMALL_WD = 3;
+constexpr int PLAN_HIST_WORDS = 4096;  // key histogram of the plan kernels (>= number of keys)  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {
@@ -121,6 +124,11 @@ struct f2_store {
     int32_t* rep_list;      // per-row scratch of pass 1 (capacity rep_capacity rows)
     int32_t* rep_dup;
     int64_t rep_capacity;
+    // per-context scratch of the full-rank check: chunks claimed [C], chunks
+    // done [C], contradiction count [C], first contradicting row [C]
+    int* full_ctr;
+    unsigned long long* full_cnt;
+    unsigned long long* full_first;
     // scratch of f2_encode_batched (grouping of the queries by context)
     mutable int32_t* enc_bins;              // bucket sizes / starts, tile sums, ticket
     mutable int64_t enc_bin_cap;

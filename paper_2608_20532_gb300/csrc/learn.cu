@@ -981,6 +981,7 @@ __global__ void __launch_bounds__(WIDE_WARPS * 32) elim_wide_kernel(StoreDev s, 
 //     warp, CTA or wide elimination queue.
 constexpr int PLAN_SUB = PLAN_BUCKETS * NARROW_WD;  // (bucket, width) keys per class
 constexpr int PLAN_KEYS = NUM_CLASSES * PLAN_SUB;
+static_assert(PLAN_KEYS <= PLAN_HIST_WORDS, "the plan histogram holds every key");
 
 struct PlanArgs {
     const int64_t* row_off;
@@ -1018,7 +1019,9 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
             if (!ok) record_status(s.status, F2_ERR_ROWS);
             R = ok ? rows : -1;
             if (p.mode == 0 && p.rep_count) {
-                if (R > 0 && cd.xw > DD_XW) {
+                // wide rows are not deduplicated; rows of a full-rank context
+                // are checked one by one (verify_full_kernel)
+                if (R > 0 && (cd.xw > DD_XW || s.rank[c] == cd.d)) {
                     p.rep_count[c] = (int32_t)(-(R + 2));
                     R = 0;
                 } else {
@@ -1036,7 +1039,8 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
             } else {
                 const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
                                    R * cd.d > p.warp_work;
-                if (cd.wd > NARROW_WD) cls = CLS_WIDE;
+                if (s.rank[c] == cd.d) cls = CLS_FULL;
+                else if (cd.wd > NARROW_WD) cls = CLS_WIDE;
                 else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
                 else cls = heavy ? CLS_CTA : CLS_WARP;
                 work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
@@ -1132,9 +1136,194 @@ int launch_plan(const StoreDev& sd, const PlanArgs& pa, int num_sms, cudaStream_
 inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) == 0; }
 
 // Shared-memory need of the narrow elimination kernel for a set of widths.
+// ---------------------------------------------------------------------------
+// Full-rank contexts.  When rank = d at the start of a call the reduced basis
+// is the identity (every coordinate is a pivot and a reduced row has no other
+// pivot bit), so every row lies in the span and T(q) = XOR of z_k over the set
+// coordinates k of q.  A row is redundant if its word equals T(phi(x)) and a
+// contradiction otherwise (Sec. 2.2 steps (2)-(3)); nothing is inserted, so
+// the rows are independent.  CTAs claim chunks of FULL_CHUNK rows of a
+// context, look T up in a 4-bit table of the z_k in shared memory (built when
+// a CTA moves to a context: entry 16p + v = XOR of z_{4p+b} over the bits b
+// of v), and the last chunk of a context commits the contradiction count,
+// the first contradicting row and rows_seen.
+// ---------------------------------------------------------------------------
+constexpr int FULL_THREADS = 256;
+constexpr int FULL_CHUNK = 2048;   // rows claimed at a time
+constexpr int FULL_STAGE = FULL_THREADS;  // rows staged in shared memory at a time (one per thread)
+
+struct FullArgs {
+    const int64_t* row_off;
+    const int64_t* x_off;
+    const uint32_t* x;
+    const uint4* y;
+    const int32_t* queue;
+    const int* counters;
+    int* ctr;                         // [2C]: chunks claimed, chunks done
+    unsigned long long* cnt;          // [C] contradicting rows of the call
+    unsigned long long* first;        // [C] first contradicting row of the call (all ones: none)
+    int table_words;                  // >= 64 * ceil(d / 4) for every context
+};
+
+__global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, FullArgs a)
+{
+    extern __shared__ uint4 full_smem[];
+    uint32_t* const tabw = reinterpret_cast<uint32_t*>(full_smem);
+    uint32_t* const stage = tabw + a.table_words;
+    __shared__ int s_q, s_k;
+    __shared__ unsigned long long s_cnt, s_first;
+    const int t = threadIdx.x, lane = t & 31;
+    const int nq = a.counters[CNT_COUNT + CLS_FULL];
+    const int qb = a.counters[CNT_BEGIN + CLS_FULL];
+    int q = 0, built = -1;
+    for (;;) {
+        if (t == 0) {
+            int k = 0;
+            while (q < nq) {
+                const int c = a.queue[qb + q];
+                const int64_t T = a.row_off[c + 1] - a.row_off[c];
+                k = atomicAdd(a.ctr + c, 1);
+                if ((int64_t)k * FULL_CHUNK < T) break;
+                ++q;
+            }
+            s_q = q;
+            s_k = k;
+            s_cnt = 0ull;
+            s_first = ~0ull;
+        }
+        __syncthreads();
+        q = s_q;
+        if (q >= nq) break;
+        const int k = s_k;
+        const int c = a.queue[qb + q];
+        const CtxDesc cd = s.desc[c];
+        const int np = (cd.d + 3) >> 2;
+        uint2* Zl = reinterpret_cast<uint2*>(tabw);
+        uint2* Zh = Zl + np * 16;
+        if (built != c) {
+            for (int j = t; j < 4 * np; j += FULL_THREADS) {
+                const uint4 z = (j < cd.d) ? __ldg(s.bz + cd.slot_off + j) : make_uint4(0, 0, 0, 0);
+                const int e = (j >> 2) * 16 + (1 << (j & 3));
+                Zl[e] = make_uint2(z.x, z.y);
+                Zh[e] = make_uint2(z.z, z.w);
+                if ((j & 3) == 0) {
+                    Zl[e - 1] = make_uint2(0, 0);
+                    Zh[e - 1] = make_uint2(0, 0);
+                }
+            }
+            __syncthreads();
+            for (int f = t; f < 16 * np; f += FULL_THREADS) {
+                const int v = f & 15;
+                if (__popc(v) < 2) continue;
+                const int eb = f & ~15;
+                uint2 lo = make_uint2(0, 0), hi = make_uint2(0, 0);
+#pragma unroll
+                for (int bb = 0; bb < 4; ++bb) {
+                    if ((v >> bb) & 1) {
+                        const uint2 l = Zl[eb + (1 << bb)], h = Zh[eb + (1 << bb)];
+                        lo.x ^= l.x;
+                        lo.y ^= l.y;
+                        hi.x ^= h.x;
+                        hi.y ^= h.y;
+                    }
+                }
+                Zl[f] = lo;
+                Zh[f] = hi;
+            }
+            built = c;
+        }
+        const int64_t r0 = a.row_off[c];
+        const int64_t T = a.row_off[c + 1] - r0;
+        const int64_t i0 = (int64_t)k * FULL_CHUNK;
+        const int64_t i1 = (i0 + FULL_CHUNK < T) ? i0 + FULL_CHUNK : T;
+        const uint32_t* xc = a.x + a.x_off[c];
+        const int xw = cd.xw;
+        const int sst = xw | 1;  // odd staging stride: a row per lane reads distinct banks
+        const uint32_t lm = (cd.n & 31) ? (1u << (cd.n & 31)) - 1u : 0xFFFFFFFFu;
+        unsigned long long cnt = 0ull, first = ~0ull;
+        for (int64_t b0 = i0; b0 < i1; b0 += FULL_STAGE) {
+            const int nb = (int)((i1 - b0) < FULL_STAGE ? (i1 - b0) : FULL_STAGE);
+            __syncthreads();  // the table is complete / the previous rows are consumed
+            const uint32_t* src = xc + b0 * xw;  // the rows are contiguous
+            for (int w = t; w < nb * xw; w += FULL_THREADS) {
+                const int r = w / xw;
+                stage[r * sst + (w - r * xw)] = __ldg(src + w);
+            }
+            __syncthreads();
+            if (t < nb) {
+                const int64_t i = b0 + t;
+                const uint4 yi = __ldg(a.y + r0 + i);
+                const uint32_t* xr = stage + t * sst;
+                uint32_t a0 = 0, a1 = 0, a2 = 0, a3 = 0, prev = 0;
+                const uint2* zl = Zl;
+                const uint2* zh = Zh;
+                for (int w = 0, left = np; left > 0; ++w, left -= 8, zl += 128, zh += 128) {
+                    uint32_t xv = (w < xw) ? xr[w] : 0u;
+                    if (w == xw - 1) xv &= lm;
+                    uint32_t qw;
+                    if (s.raw) {
+                        qw = xv;
+                    } else {  // phi(x) = [1 || x]: the constant at index 0, x bit j at 1 + j
+                        qw = (xv << 1) | (prev >> 31) | (w == 0 ? 1u : 0u);
+                        prev = xv;
+                    }
+#pragma unroll
+                    for (int h = 0; h < 8; ++h) {
+                        if (h < left) {
+                            const int e = h * 16 + (int)((qw >> (4 * h)) & 15u);
+                            const uint2 lo = zl[e], hi = zh[e];
+                            a0 ^= lo.x;
+                            a1 ^= lo.y;
+                            a2 ^= hi.x;
+                            a3 ^= hi.y;
+                        }
+                    }
+                }
+                if (a0 != yi.x || a1 != yi.y || a2 != yi.z || a3 != yi.w) {
+                    ++cnt;
+                    if ((unsigned long long)i < first) first = (unsigned long long)i;
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            cnt += __shfl_xor_sync(FULL, cnt, o);
+            const unsigned long long f2 = __shfl_xor_sync(FULL, first, o);
+            first = f2 < first ? f2 : first;
+        }
+        if (lane == 0 && cnt) {
+            atomicAdd(&s_cnt, cnt);
+            atomicMin(&s_first, first);
+        }
+        __syncthreads();
+        if (t == 0) {
+            if (s_cnt) {
+                atomicAdd(a.cnt + c, s_cnt);
+                atomicMin(a.first + c, s_first);
+            }
+            __threadfence();
+            const int nch = (int)((T + FULL_CHUNK - 1) / FULL_CHUNK);
+            if (atomicAdd(a.ctr + s.num_ctx + c, 1) == nch - 1) {  // the context's last chunk
+                __threadfence();
+                const unsigned long long tot = atomicAdd(a.cnt + c, 0ull);
+                const unsigned long long fi = atomicMin(a.first + c, ~0ull);
+                const long long seen = s.rows_seen[c];
+                if (tot) {
+                    s.n_contra[c] += tot;
+                    s.contra[c] = 1;
+                    if (s.first_contra[c] < 0) s.first_contra[c] = seen + (long long)fi;
+                }
+                s.rows_seen[c] = seen + T;
+            }
+        }
+        __syncthreads();
+    }
+}
+
 // Which elimination kernels a store needs, and their widest bases.
 struct Widths {
     int max_small_words = 0, max_narrow_words = 0, max_wide_d = 0;
+    int max_d = 0, max_xw = 0;  // over every context (any may reach full rank)
     bool has_small = false, has_narrow = false, has_wide = false;
 };
 
@@ -1149,7 +1338,8 @@ size_t narrow_smem(int max_narrow_words, int warp_region_words)
 int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* row_off, const int64_t* x_off,
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
-                       const Widths& wv, cudaStream_t cs)
+                       const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
+                       unsigned long long* full_first, cudaStream_t cs)
 {
     PlanArgs pa;
     pa.row_off = row_off;
@@ -1188,6 +1378,34 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words));
         if (rc != F2_OK) return rc;
     }
+    {  // full-rank contexts (the plan decides on the device which, if any)
+        const int C = sd.num_ctx;
+        e = cudaMemsetAsync(full_ctr, 0, sizeof(int) * 2 * (size_t)C, cs);
+        if (e == cudaSuccess) e = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
+        if (e == cudaSuccess) e = cudaMemsetAsync(full_first, 0xff, sizeof(unsigned long long) * (size_t)C, cs);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        FullArgs fa;
+        fa.row_off = row_off;
+        fa.x_off = x_off;
+        fa.x = la.x;
+        fa.y = la.y;
+        fa.queue = queue;
+        fa.counters = la.counters;
+        fa.ctr = full_ctr;
+        fa.cnt = full_cnt;
+        fa.first = full_first;
+        fa.table_words = 64 * ((wv.max_d + 3) / 4);
+        const size_t smem = 4 * ((size_t)fa.table_words + (size_t)FULL_STAGE * (size_t)(wv.max_xw | 1));
+        e = cudaFuncSetAttribute(verify_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        int per_sm = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_full_kernel, FULL_THREADS, smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        if (per_sm < 1) per_sm = 1;
+        verify_full_kernel<<<num_sms * per_sm, FULL_THREADS, smem, cs>>>(sd, fa);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
     if (wv.has_wide) {
         const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
         e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -1206,6 +1424,8 @@ Widths width_summary(const int32_t* n_bits, int32_t num_ctx, bool raw)
         const int d = raw ? n_bits[c] : n_bits[c] + 1;
         const int wd = (d + 31) / 32;
         const int words = elim_words(d, wd);
+        if (d > w.max_d) w.max_d = d;
+        if ((n_bits[c] + 31) / 32 > w.max_xw) w.max_xw = (n_bits[c] + 31) / 32;
         if (wd <= SMALL_WD) {
             w.has_small = true;
             if (words > w.max_small_words) w.max_small_words = words;
@@ -1292,7 +1512,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     const Widths wv = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
-                              wv, cs);
+                              wv, st->full_ctr, st->full_cnt, st->full_first, cs);
 }
 
 // ---------------------------------------------------------------------------
@@ -1309,8 +1529,11 @@ struct NoallocScratch {
     int32_t n_bits[F2_NOALLOC_MAX_CTX];
     int32_t queue[F2_NOALLOC_MAX_CTX];
     int32_t keybuf[F2_NOALLOC_MAX_CTX];
-    int counters[32];
+    int counters[CNT_WORDS];
     int plan_hist[PLAN_KEYS];
+    int full_ctr[2 * F2_NOALLOC_MAX_CTX];
+    unsigned long long full_cnt[F2_NOALLOC_MAX_CTX];
+    unsigned long long full_first[F2_NOALLOC_MAX_CTX];
 };
 
 // Device storage for the scratch; in host code this name is only a symbol
@@ -1492,5 +1715,6 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
     const Widths wv = width_summary(n_bits_host, num_ctx, raw);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,
-                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, sc->plan_hist, nd->num_sms, wv, cs);
+                              DEFAULT_WARP_WORK, sc->queue, sc->keybuf, sc->plan_hist, nd->num_sms, wv, sc->full_ctr,
+                              sc->full_cnt, sc->full_first, cs);
 }

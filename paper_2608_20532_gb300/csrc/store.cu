@@ -40,6 +40,7 @@ static void free_store(f2_store* s)
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
+                    s->full_ctr, s->full_cnt, s->full_first,
                     s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items};
     for (void* p : ptrs)
         if (p) cudaFree(p);
@@ -134,7 +135,10 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     alloc((void**)&s->keybuf, sizeof(int32_t) * C);
     alloc((void**)&s->counters, sizeof(int) * CNT_WORDS);
     alloc((void**)&s->rep_count, sizeof(int32_t) * C);
-    alloc((void**)&s->plan_hist, sizeof(int) * 4096);
+    alloc((void**)&s->plan_hist, sizeof(int) * PLAN_HIST_WORDS);
+    alloc((void**)&s->full_ctr, sizeof(int) * 2 * C);
+    alloc((void**)&s->full_cnt, sizeof(unsigned long long) * C);
+    alloc((void**)&s->full_first, sizeof(unsigned long long) * C);
     cudaStream_t st = (cudaStream_t)stream;
     if (e == cudaSuccess && num_ctx)
         e = cudaMemcpyAsync(s->desc, desc.data(), sizeof(CtxDesc) * (size_t)num_ctx,
