@@ -125,7 +125,9 @@ struct f2_store {
     int32_t* rep_dup;
     int64_t rep_capacity;
     // per-context scratch of the full-rank check: chunks claimed [C], chunks
-    // done [C], contradiction count [C], first contradicting row [C]
+    // done [C], first row left and list of the contexts that reached full rank
+    // during a call [C each] and their count; contradiction count [C], first
+    // contradicting row [C]
     int* full_ctr;
     unsigned long long* full_cnt;
     unsigned long long* full_first;

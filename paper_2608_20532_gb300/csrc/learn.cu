@@ -56,6 +56,11 @@ struct LearnArgs {
     const int32_t* queue;
     int* counters;
     int warp_region_words;
+    // contexts that reach full rank with rows left (not deduplicated): listed
+    // here, the rest of their rows checked by verify_full_kernel
+    int* late_count;
+    int32_t* late_list;
+    int32_t* late_start;
 };
 
 struct DedupArgs {
@@ -78,6 +83,9 @@ constexpr int CTL_RANK = 160;  // rank
 constexpr int CTL_CNT = 162;   // contradiction count (uint64, 8-byte aligned)
 constexpr int CTL_FIRST = 164; // first contradiction index (int64)
 constexpr int CTL_WORDS = 176; // size of the control area (16-byte multiple)
+
+constexpr int FULL_THREADS = 1024;  // verify_full_kernel: one table shared by 32 warps
+constexpr int FULL_CHUNK = 2048;   // rows of a full-rank context claimed at a time
 
 // Pass 1: 16 warps per CTA, one CTA per SM.  A warp-owned context (at most
 // DD_WARP_MAX_ROWS rows) gets a table of next_pow2(2T) entries in a 12 KB
@@ -814,6 +822,7 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     uint32_t xn[WD];
     uint4 yn;
     load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
+    int stop_at = -1;
     for (int base = 0; base < R; base += nt) {
         const bool valid = nvalid;
         const int i = ni;
@@ -876,6 +885,15 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
             if (CTA) {
                 if (t < 48) NPR[t] = 0u;
             }
+            // (wide contexts) full rank with at least a chunk of rows left:
+            // every later row is a check only (the rows are their own
+            // representatives here)
+            if constexpr (WD > NARROW_WD) {
+                if (!deduped && a.late_list && R - (base + nt) >= FULL_CHUNK && *rank_s == cd.d) {
+                    stop_at = base + nt;
+                    break;
+                }
+            }
         }
         (void)contra_lane;
     }
@@ -889,8 +907,13 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     basis_from_smem<WD>(s, cd, S, t, nt);
     if (t == 0) {
         s.rank[c] = *rank_s;
-        s.rows_seen[c] = seen + T;
         commit_stats(s, c, *first_s, *cnt_s);
+        if (stop_at < 0) {
+            s.rows_seen[c] = seen + T;
+        } else {  // rows_seen is advanced by verify_full_kernel
+            a.late_start[c] = stop_at;
+            a.late_list[atomicAdd(a.late_count, 1)] = c;
+        }
     }
     group_sync<CTA>();
 }
@@ -1148,8 +1171,6 @@ inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) ==
 // of v), and the last chunk of a context commits the contradiction count,
 // the first contradicting row and rows_seen.
 // ---------------------------------------------------------------------------
-constexpr int FULL_THREADS = 256;
-constexpr int FULL_CHUNK = 2048;   // rows claimed at a time
 constexpr int FULL_STAGE = FULL_THREADS;  // rows staged in shared memory at a time (one per thread)
 
 struct FullArgs {
@@ -1160,6 +1181,9 @@ struct FullArgs {
     const int32_t* queue;
     const int* counters;
     int* ctr;                         // [2C]: chunks claimed, chunks done
+    const int* late_count;            // contexts listed by the elimination kernels
+    const int32_t* late_list;
+    const int32_t* late_start;        // their first row left
     unsigned long long* cnt;          // [C] contradicting rows of the call
     unsigned long long* first;        // [C] first contradicting row of the call (all ones: none)
     int table_words;                  // >= 64 * ceil(d / 4) for every context
@@ -1173,15 +1197,18 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
     __shared__ int s_q, s_k;
     __shared__ unsigned long long s_cnt, s_first;
     const int t = threadIdx.x, lane = t & 31;
-    const int nq = a.counters[CNT_COUNT + CLS_FULL];
+    const int nfull = a.counters[CNT_COUNT + CLS_FULL];
     const int qb = a.counters[CNT_BEGIN + CLS_FULL];
+    const int nq = nfull + *a.late_count;  // full at the start of the call, then full mid-call
+    auto ctx_of = [&](int qq) { return qq < nfull ? a.queue[qb + qq] : a.late_list[qq - nfull]; };
+    auto start_of = [&](int qq, int c) { return qq < nfull ? (int64_t)0 : (int64_t)a.late_start[c]; };
     int q = 0, built = -1;
     for (;;) {
         if (t == 0) {
             int k = 0;
             while (q < nq) {
-                const int c = a.queue[qb + q];
-                const int64_t T = a.row_off[c + 1] - a.row_off[c];
+                const int c = ctx_of(q);
+                const int64_t T = a.row_off[c + 1] - a.row_off[c] - start_of(q, c);
                 k = atomicAdd(a.ctr + c, 1);
                 if ((int64_t)k * FULL_CHUNK < T) break;
                 ++q;
@@ -1195,7 +1222,8 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
         q = s_q;
         if (q >= nq) break;
         const int k = s_k;
-        const int c = a.queue[qb + q];
+        const int c = ctx_of(q);
+        const int64_t i_first = start_of(q, c);
         const CtxDesc cd = s.desc[c];
         const int np = (cd.d + 3) >> 2;
         uint2* Zl = reinterpret_cast<uint2*>(tabw);
@@ -1234,7 +1262,7 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
         }
         const int64_t r0 = a.row_off[c];
         const int64_t T = a.row_off[c + 1] - r0;
-        const int64_t i0 = (int64_t)k * FULL_CHUNK;
+        const int64_t i0 = i_first + (int64_t)k * FULL_CHUNK;
         const int64_t i1 = (i0 + FULL_CHUNK < T) ? i0 + FULL_CHUNK : T;
         const uint32_t* xc = a.x + a.x_off[c];
         const int xw = cd.xw;
@@ -1245,9 +1273,20 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
             const int nb = (int)((i1 - b0) < FULL_STAGE ? (i1 - b0) : FULL_STAGE);
             __syncthreads();  // the table is complete / the previous rows are consumed
             const uint32_t* src = xc + b0 * xw;  // the rows are contiguous
-            for (int w = t; w < nb * xw; w += FULL_THREADS) {
-                const int r = w / xw;
-                stage[r * sst + (w - r * xw)] = __ldg(src + w);
+            {
+                // word w = r * xw + v of the block, stepped by FULL_THREADS
+                // without a division per word
+                int r = t / xw, v = t - (t / xw) * xw;
+                const int dr = FULL_THREADS / xw, dv = FULL_THREADS - dr * xw;
+                for (int w = t; w < nb * xw; w += FULL_THREADS) {
+                    stage[r * sst + v] = __ldg(src + w);
+                    r += dr;
+                    v += dv;
+                    if (v >= xw) {
+                        v -= xw;
+                        ++r;
+                    }
+                }
             }
             __syncthreads();
             if (t < nb) {
@@ -1302,7 +1341,7 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
                 atomicMin(a.first + c, s_first);
             }
             __threadfence();
-            const int nch = (int)((T + FULL_CHUNK - 1) / FULL_CHUNK);
+            const int nch = (int)((T - i_first + FULL_CHUNK - 1) / FULL_CHUNK);
             if (atomicAdd(a.ctr + s.num_ctx + c, 1) == nch - 1) {  // the context's last chunk
                 __threadfence();
                 const unsigned long long tot = atomicAdd(a.cnt + c, 0ull);
@@ -1341,6 +1380,17 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
                        unsigned long long* full_first, cudaStream_t cs)
 {
+    // full_ctr: chunks claimed [C], chunks done [C], late start [C], late list [C], late count
+    const int C = sd.num_ctx;
+    LearnArgs lx = la;
+    lx.late_start = full_ctr + 2 * C;
+    lx.late_list = full_ctr + 3 * C;
+    lx.late_count = full_ctr + 4 * C;
+    {
+        cudaError_t e0 = cudaMemsetAsync(full_ctr, 0, sizeof(int) * 2 * (size_t)C, cs);
+        if (e0 == cudaSuccess) e0 = cudaMemsetAsync(lx.late_count, 0, sizeof(int), cs);
+        if (e0 != cudaSuccess) return f2_cuda_status(e0);
+    }
     PlanArgs pa;
     pa.row_off = row_off;
     pa.x_off = x_off;
@@ -1365,7 +1415,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, LEARN_WARPS * 32, smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         if (per_sm < 1) per_sm = 1;
-        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, la);
+        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, lx);
         return f2_cuda_status(cudaGetLastError());
     };
     if (wv.has_small) {
@@ -1378,10 +1428,17 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words));
         if (rc != F2_OK) return rc;
     }
-    {  // full-rank contexts (the plan decides on the device which, if any)
-        const int C = sd.num_ctx;
-        e = cudaMemsetAsync(full_ctr, 0, sizeof(int) * 2 * (size_t)C, cs);
-        if (e == cudaSuccess) e = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
+    if (wv.has_wide) {
+        const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
+        e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, cs>>>(sd, lx);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    {  // full-rank contexts: at the start of the call (the plan decides on the
+       // device which, if any) or reached during it (listed by the kernels above)
+        e = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
         if (e == cudaSuccess) e = cudaMemsetAsync(full_first, 0xff, sizeof(unsigned long long) * (size_t)C, cs);
         if (e != cudaSuccess) return f2_cuda_status(e);
         FullArgs fa;
@@ -1392,6 +1449,9 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         fa.queue = queue;
         fa.counters = la.counters;
         fa.ctr = full_ctr;
+        fa.late_count = lx.late_count;
+        fa.late_list = lx.late_list;
+        fa.late_start = lx.late_start;
         fa.cnt = full_cnt;
         fa.first = full_first;
         fa.table_words = 64 * ((wv.max_d + 3) / 4);
@@ -1403,14 +1463,6 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         if (e != cudaSuccess) return f2_cuda_status(e);
         if (per_sm < 1) per_sm = 1;
         verify_full_kernel<<<num_sms * per_sm, FULL_THREADS, smem, cs>>>(sd, fa);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
-    }
-    if (wv.has_wide) {
-        const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
-        e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, cs>>>(sd, la);
         e = cudaGetLastError();
         if (e != cudaSuccess) return f2_cuda_status(e);
     }
@@ -1531,7 +1583,7 @@ struct NoallocScratch {
     int32_t keybuf[F2_NOALLOC_MAX_CTX];
     int counters[CNT_WORDS];
     int plan_hist[PLAN_KEYS];
-    int full_ctr[2 * F2_NOALLOC_MAX_CTX];
+    int full_ctr[4 * F2_NOALLOC_MAX_CTX + 1];
     unsigned long long full_cnt[F2_NOALLOC_MAX_CTX];
     unsigned long long full_first[F2_NOALLOC_MAX_CTX];
 };

@@ -136,7 +136,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     alloc((void**)&s->counters, sizeof(int) * CNT_WORDS);
     alloc((void**)&s->rep_count, sizeof(int32_t) * C);
     alloc((void**)&s->plan_hist, sizeof(int) * PLAN_HIST_WORDS);
-    alloc((void**)&s->full_ctr, sizeof(int) * 2 * C);
+    alloc((void**)&s->full_ctr, sizeof(int) * (4 * C + 1));
     alloc((void**)&s->full_cnt, sizeof(unsigned long long) * C);
     alloc((void**)&s->full_first, sizeof(unsigned long long) * C);
     cudaStream_t st = (cudaStream_t)stream;
