@@ -39,6 +39,7 @@ EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
     "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3", "f2_learn_batched_noalloc",
+    "f2_encode_epilogue",
 )
 
 _lib = None
@@ -76,6 +77,7 @@ def load_library(path: Optional[str] = None):
         "f2_get_basis": ([P] + [P] * 8 + [P], ctypes.c_int),
         "f2_solve_affine": ([P, P, P], ctypes.c_int),
         "f2_encode_batched": ([P, i64, P, P, i32, P, P, P], ctypes.c_int),
+        "f2_encode_epilogue": ([P, i64, P, P, P, P, P, P, P], ctypes.c_int),
         "f2_device_status": ([P, ctypes.POINTER(ctypes.c_int), P], ctypes.c_int),
         "f2_store_export": ([P, P, ctypes.POINTER(ctypes.c_size_t), P], ctypes.c_int),
         "f2_store_import": ([P, P, ctypes.c_size_t, P], ctypes.c_int),
@@ -205,6 +207,19 @@ class Store:
         _check(self._lib.f2_encode_batched(self._h, Q, _dptr(ctx_id), _dptr(x), stride, _dptr(y_out),
                                            _dptr(in_span), _stream(stream)), "f2_encode_batched")
         return y_out, in_span
+
+    def encode_epilogue(self, ctx_id: torch.Tensor, in_span: torch.Tensor, y: torch.Tensor, sched=None,
+                        state=None, opaque_mask=None, stream=None):
+        """Full words in place (Appendix C/D): y ^= sched << 105, then the bits
+        of opaque_mask[ctx] taken from state; rejected queries untouched.
+        sched int32[Q], state int32[Q, 4], opaque_mask int32[num_ctx, 4]."""
+        Q = int(ctx_id.numel())
+        _check(self._lib.f2_encode_epilogue(self._h, Q, _dptr(ctx_id), _dptr(in_span),
+                                            _dptr(sched) if sched is not None else None,
+                                            _dptr(state) if state is not None else None,
+                                            _dptr(opaque_mask) if opaque_mask is not None else None,
+                                            _dptr(y), _stream(stream)), "f2_encode_epilogue")
+        return y
 
     def device_status(self, stream=None) -> int:
         v = ctypes.c_int(0)

@@ -1112,5 +1112,58 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
     return F2_OK;
 }
 
+namespace {
+
+// Appendix C / D epilogue, one thread per query in query order (coalesced:
+// the caller's control and state arrays are in query order too).
+constexpr int SC_SHIFT = 105;   // scheduler control: bits 105..121 of the word
+constexpr uint32_t SC_MASK = (1u << 17) - 1u;
+
+__global__ void __launch_bounds__(256) epilogue_kernel(int64_t Q, int32_t num_ctx, const int32_t* __restrict__ ctx_id,
+                                                       const uint8_t* __restrict__ in_span,
+                                                       const uint32_t* __restrict__ sc,
+                                                       const uint4* __restrict__ state,
+                                                       const uint4* __restrict__ mask, uint4* __restrict__ y)
+{
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < Q; q += (int64_t)gridDim.x * blockDim.x) {
+        if (__ldg(in_span + q) != 1) continue;
+        uint4 w = y[q];
+        if (sc) {
+            // bits 105..121 = bits 9..25 of word 3
+            w.w ^= (__ldg(sc + q) & SC_MASK) << (SC_SHIFT - 96);
+        }
+        if (state && mask) {
+            const int32_t c = __ldg(ctx_id + q);
+            if (c >= 0 && c < num_ctx) {
+                const uint4 m = __ldg(mask + c), h = __ldg(state + q);
+                w.x = (w.x & ~m.x) | (h.x & m.x);
+                w.y = (w.y & ~m.y) | (h.y & m.y);
+                w.z = (w.z & ~m.z) | (h.z & m.z);
+                w.w = (w.w & ~m.w) | (h.w & m.w);
+            }
+        }
+        y[q] = w;
+    }
+}
+
+}  // namespace
+
+extern "C" int f2_encode_epilogue(const f2_store* st, int64_t Q, const int32_t* ctx_id, const uint8_t* in_span,
+                                  const uint32_t* sc, const uint32_t* state, const uint32_t* opaque_mask,
+                                  uint32_t* y, f2_stream_t stream)
+{
+    if (!st || Q < 0) return F2_ERR_INVALID_ARG;
+    if (Q == 0) return F2_OK;
+    if (!y || !in_span || !ctx_id) return F2_ERR_INVALID_ARG;
+    if (((uintptr_t)y % 16) != 0 || ((uintptr_t)state % 16) != 0 || ((uintptr_t)opaque_mask % 16) != 0)
+        return F2_ERR_ALIGN;
+    int64_t blocks = (Q + 255) / 256;
+    if (blocks > (int64_t)st->num_sms * 16) blocks = (int64_t)st->num_sms * 16;
+    epilogue_kernel<<<(int)blocks, 256, 0, (cudaStream_t)stream>>>(
+        Q, st->num_ctx, ctx_id, in_span, sc, reinterpret_cast<const uint4*>(state),
+        reinterpret_cast<const uint4*>(opaque_mask), reinterpret_cast<uint4*>(y));
+    return f2_cuda_status(cudaGetLastError());
+}
+
 int f2_encode_table_min_default() { return DEFAULT_TABLE_MIN; }
 int f2_encode_table_min_floor() { return RUN_SEG / MAX_TRUNS; }

@@ -171,3 +171,78 @@ def test_zipf_config3_scaled_table_mins(env):
     gpu_learn_workload(binding, st, wl, dev)
     O = oracle_for(wl)
     _compare(binding, st, O, wl.queries.ctx_id, wl.queries.x)
+
+
+def test_epilogue_appendix_c_on_gpu(env, golden_dir):
+    """The Appendix C instruction end to end on the GPU: learn the five stored
+    pairs of Table 6, encode the parsed values, merge scheduler control."""
+    import json
+    import os
+
+    from oracle import f2_bigint as bi
+
+    binding, dev = env
+    with open(os.path.join(golden_dir, "appendix_c_hmma.json")) as f:
+        g = json.load(f)
+    d = g["feature_width"]
+
+    def idx(t):
+        return 0 if t == "const" else 1 + 64 * t[0] + t[1]
+
+    rows = [(sum(1 << idx(t) for t in r["features"]), int(r["z"], 16)) for r in g["basis_rows"]]
+    nw = (d + 31) // 32
+    x = np.array([bi.int_to_words(r, nw) for r, _ in rows], np.uint32).reshape(-1)
+    y = np.array([bi.int_to_words(z, 4) for _, z in rows], np.uint32)
+    st = binding.Store([d], raw=True, device=dev)
+    rt, xot, xt, yt = dev_arrays(binding, dev, np.array([0, 5], np.int64), np.array([0], np.int64), x, y)
+    st.learn(rt, xt, xot, yt)
+    f = bi.parsed_value_features(g["values"])
+    ct, qt = dev_arrays(binding, dev, np.zeros(1, np.int32), np.array([bi.int_to_words(f, nw)], np.uint32))
+    yq, ok = st.encode(ct, qt)
+    sc = binding.to_device(np.array([int(g["sched_control"], 16)], np.int32), dev)
+    st.encode_epilogue(ct, ok, yq, sched=sc)
+    torch.cuda.synchronize()
+    words = binding.to_numpy(yq).view(np.uint32)[0]
+    assert bi.words_to_int(words) == int(g["y_full"], 16)
+    assert words.astype("<u4").tobytes().hex(" ") == g["le_bytes"]
+
+
+def test_epilogue_random(env):
+    """Random control bits, recorded states and per-context opaque masks (the
+    Appendix D mask, random masks, none) against the oracle's epilogue."""
+    from oracle import f2_bigint as bi
+
+    binding, dev = env
+    wl = wlmod.generate(wlmod.scaled(3, 300), 77, query_count=30000)
+    st = binding.Store(wl.n_bits, device=dev)
+    gpu_learn_workload(binding, st, wl, dev)
+    O = oracle_for(wl)
+    q = wl.queries
+    rng = np.random.default_rng(5)
+    Q = len(q.ctx_id)
+    ctx = q.ctx_id.copy()
+    ctx[::997] = wl.num_ctx + 3  # a few bad ids: rejected, untouched
+    sched = rng.integers(0, 2 ** 31, size=Q, dtype=np.int64).astype(np.int32)
+    state = rng.integers(0, 2 ** 32, size=(Q, 4), dtype=np.uint64).astype(np.uint32)
+    masks = np.zeros((wl.num_ctx, 4), np.uint32)
+    masks[::3, 3] = (1 << (122 - 96)) | (1 << (124 - 96))
+    masks[1::3] = rng.integers(0, 2 ** 32, size=masks[1::3].shape, dtype=np.uint64).astype(np.uint32)
+    ry, rok = O.encode(ctx, q.x)
+    ct, xt = dev_arrays(binding, dev, ctx, q.x)
+    yq, ok = st.encode(ct, xt)
+    for variant in ("all", "no_state", "no_sched"):
+        y2 = yq.clone()
+        st.encode_epilogue(ct, ok, y2, sched=None if variant == "no_sched" else binding.to_device(sched, dev),
+                           state=None if variant == "no_state" else binding.to_device(state, dev),
+                           opaque_mask=binding.to_device(masks, dev))
+        torch.cuda.synchronize()
+        got = binding.to_numpy(y2).view(np.uint32)
+        assert np.array_equal(binding.to_numpy(ok), rok)
+        for i in range(0, Q, 7):
+            c = int(ctx[i])
+            m = bi.words_to_int(masks[c]) if (0 <= c < wl.num_ctx and variant != "no_state") else 0
+            want = bi.encode_epilogue(bi.words_to_int(ry[i]), rok[i] == 1,
+                                      sched=0 if variant == "no_sched" else int(sched[i]) & 0xFFFFFFFF,
+                                      state=bi.words_to_int(state[i]), mask=m)
+            assert bi.words_to_int(got[i]) == want, (variant, i)
+    st.device_status()

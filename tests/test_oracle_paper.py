@@ -203,3 +203,34 @@ def test_appendix_d_bits(golden_dir):
     x = wa ^ wb
     bits = [i for i in range(128) if (int(x[i // 32]) >> (i % 32)) & 1]
     assert bits == g["xor_bits"]
+
+
+# ------------------------------------------------------- encode epilogue
+
+def test_epilogue_appendix_c(golden_dir):
+    """Eq. hmma-full-word: the learned word XOR (sc << 105), emitted as the
+    16 little-endian bytes the paper prints."""
+    g = _load(golden_dir, "appendix_c_hmma.json")
+    y_learned = _hex128(g["y_learned"])
+    full = bi.encode_epilogue(y_learned, True, sched=int(g["sched_control"], 16))
+    assert full == _hex128(g["y_full"])
+    le = np.array(bi.int_to_words(full, 4), np.uint32).astype("<u4").tobytes()
+    assert le.hex(" ") == g["le_bytes"]
+    assert bi.encode_epilogue(y_learned, False, sched=int(g["sched_control"], 16)) == 0  # rejected: no word
+
+
+def test_epilogue_appendix_d(golden_dir):
+    """Appendix D: words A and B differ only in the opaque bits 122 and 124;
+    restoring them from the recorded state gives back either word."""
+    g = _load(golden_dir, "appendix_d_depbar.json")
+    a, b = _hex128(g["word_a"]), _hex128(g["word_b"])
+    mask = sum(1 << k for k in g["xor_bits"])
+    learned = a & ~mask  # the learned map excludes the masked bits
+    assert learned == b & ~mask
+    assert bi.encode_epilogue(learned, True, state=b, mask=mask) == b
+    assert bi.encode_epilogue(learned, True, state=a, mask=mask) == a
+    assert bi.encode_epilogue(a, True) == a  # no control, no mask: unchanged
+    # only the 17 control bits are merged, at 105..121, below the opaque bits
+    assert bi.encode_epilogue(0, True, sched=(1 << 17) | 1) == 1 << 105
+    assert bi.encode_epilogue(0, True, sched=(1 << 17) - 1) == ((1 << 17) - 1) << 105
+    assert ((((1 << 17) - 1) << 105) & mask) == 0
