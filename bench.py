@@ -135,6 +135,9 @@ def reduce_across_ranks(value: float, op: str, device=None) -> float:
 def workload_for(cfg_id: int, rank: int, query_count=None, num_ctx=None):
     from paper_2608_20532_gb300 import workloads as W
 
+    if cfg_id == 6:  # parsed-value contexts with the paper's low exact-context ranks
+        over = {"num_ctx": num_ctx} if num_ctx else {}
+        return W.parsed_lowrank(seed=W.seed_for(6) + 1000 * rank, **over)
     cfg = dict(W.CONFIGS[cfg_id]) if not num_ctx else W.scaled(cfg_id, num_ctx)
     if num_ctx and query_count is None and cfg.get("queries", {}).get("count"):
         query_count = int(cfg["queries"]["count"] * num_ctx / W.CONFIGS[cfg_id]["num_ctx"])
@@ -143,11 +146,13 @@ def workload_for(cfg_id: int, rank: int, query_count=None, num_ctx=None):
 
 
 def describe(cfg_id: int, wl) -> dict:
-    scaled_note = "" if wl.num_ctx == {1: 256, 2: 4096, 3: 77926, 5: 64}[cfg_id] else " [SCALED DOWN]"
+    scaled_note = "" if wl.num_ctx == {1: 256, 2: 4096, 3: 77926, 5: 64, 6: 10000}[cfg_id] else " [SCALED DOWN]"
     d = {"workload": scaled_note + {1: "config-1 parity case: 256 contexts, n=48, 260 rows each, 100 queries/context",
                       2: "4,096 contexts, n in [32,128], ~2.6M rows",
                       3: "joint-Blackwell-scale learn (77,926 contexts, ~80M rows, 85% duplicates) + 10M Zipf(1.1) encode queries",
-                      5: "64 contexts, n=1024, 2^20 rows each in 16 incremental 65,536-row batches"}[cfg_id],
+                      5: "64 contexts, n=1024, 2^20 rows each in 16 incremental 65,536-row batches",
+                      6: "parsed-value contexts: 10,000 contexts of k in [2,8] int64 values (n = 64k), exact-context "
+                         "rank median 3 / p95 21, ~200 rows per rank (13.6M rows)"}[cfg_id],
          "contexts": wl.num_ctx, "rows": wl.total_rows, "n_median": float(np.median(wl.n_bits)),
          "queries": int(len(wl.queries.ctx_id)) if wl.queries is not None else 0,
          "input_bytes": int(wl.x.nbytes + wl.y.nbytes),
@@ -510,12 +515,15 @@ def run_ours(args):
 
 def launches_per_step(wl, has_q: bool) -> int:
     """Kernels one step enqueues (the host logic of the library): per learn
-    call a plan (3 kernels) and dedup_kernel for the duplicate pass, a plan,
+    call a plan (3 kernels) and dedup_kernel (a second instance when some
+    feature row has more than 9 words) for the duplicate pass, a plan,
     the elimination kernel of each width class present (d <= 96, 96 < d <=
     288, wider) and the full-rank check; solve_kernel; per 2^25 queries the
     five encode kernels."""
     wd = (wl.n_bits.astype(np.int64) + 1 + 31) // 32
-    learn = 3 + 1 + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any()) + int(store_has_wide(wl)) + 1
+    xw = (wl.n_bits.astype(np.int64) + 31) // 32
+    learn = (3 + 1 + int((xw > 9).any()) + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any())
+             + int(store_has_wide(wl)) + 1)
     enc = 5 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
     return len(wl.batches) * learn + 1 + enc
 
@@ -676,7 +684,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, choices=[1, 2, 3, 5], default=3)
+    ap.add_argument("--config", type=int, choices=[1, 2, 3, 5, 6], default=3)
     ap.add_argument("--ctx", type=int, default=0,
                     help="scaled-down workload with this many contexts (profiling); 0 = full size")
     ap.add_argument("--e2e-steps", type=int, default=5)

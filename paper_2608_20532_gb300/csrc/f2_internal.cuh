@@ -42,11 +42,14 @@ enum Class {
     CLS_CTA_S = 6,
     CLS_WARP_S = 7,
     CLS_FULL = 8,
-    NUM_CLASSES = 9
+    CLS_DDW_CTA = 9,   // dedup of feature rows of 10..16 words (their own kernel)
+    CLS_DDW_QUAD = 10,
+    CLS_DDW_WARP = 11,
+    NUM_CLASSES = 12
 };
 static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
 constexpr int SMALL_WD = 3;
-constexpr int PLAN_HIST_WORDS = 4096;  // key histogram of the plan kernels (>= number of keys)  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
+constexpr int PLAN_HIST_WORDS = 8192;  // key histogram of the plan kernels (>= number of keys)  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {
@@ -93,6 +96,7 @@ struct f2_store {
     int device;
     int num_sms;
     int32_t max_wd;
+    int32_t max_xw;         // widest feature row (words) supplied
     int32_t max_d;
     int32_t n_wide;         // contexts with wd > NARROW_WD
     int64_t slots;

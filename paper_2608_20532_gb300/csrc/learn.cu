@@ -101,7 +101,8 @@ constexpr int DD_QUAD_E = 4 * DD_WARP_E;
 constexpr int DD_CTA_E = 16384;
 constexpr int DD_SMEM = 4 * 3 * DD_CTA_E;       // bytes (also 16 warp regions)
 constexpr int DD_K = 4;                         // rows per thread in flight
-constexpr int DD_XW = NARROW_WD;                // widest feature row (words) that is deduplicated
+constexpr int DD_XW = NARROW_WD;                // widest feature row (words) of dedup_kernel<false>
+constexpr int DD_XW_WIDE = 16;                  // widest of dedup_kernel<true> (one row in flight)
 constexpr int DEDUP_PROBES = 8;                 // linear-probe limit
 static_assert(DD_WARPS * DD_WARP_REGION * 4 <= DD_SMEM, "warp regions exceed the dedup shared memory");
 
@@ -124,6 +125,18 @@ __host__ __device__ __forceinline__ int elim_words(int d, int wd) { return CTL_W
     case 7: CALL(7); break;          \
     case 8: CALL(8); break;          \
     case 9: CALL(9); break;          \
+    default: break;                  \
+    }
+
+#define F2_XWIDE_SWITCH(wd, CALL)    \
+    switch (wd) {                    \
+    case 10: CALL(10); break;        \
+    case 11: CALL(11); break;        \
+    case 12: CALL(12); break;        \
+    case 13: CALL(13); break;        \
+    case 14: CALL(14); break;        \
+    case 15: CALL(15); break;        \
+    case 16: CALL(16); break;        \
     default: break;                  \
     }
 
@@ -322,7 +335,7 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
     int nrep = 0;
     // rows of the round in flight, and the next round's rows prefetched while
     // the current one is probed and verified
-    constexpr int K = (XW <= 2) ? DD_K : 2;
+    constexpr int K = (XW <= 2) ? DD_K : (XW <= NARROW_WD ? 2 : 1);
     uint4 yn[K];
     uint32_t xn[K][XW];
 #pragma unroll
@@ -475,18 +488,23 @@ __device__ __forceinline__ int pow2_at_least(int v)
 }
 
 // Pass 1 kernel: CTA-owned contexts first, then quads, then warps.
+template <bool WX>
 __global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupArgs a)
 {
+    // WX: the contexts whose feature rows have DD_XW + 1 .. DD_XW_WIDE words
+    constexpr int C_CTA = WX ? CLS_DDW_CTA : CLS_DD_CTA;
+    constexpr int C_QUAD = WX ? CLS_DDW_QUAD : CLS_DD_QUAD;
+    constexpr int C_WARP = WX ? CLS_DDW_WARP : CLS_DD_WARP;
     extern __shared__ __align__(16) uint32_t smem[];
     __shared__ int s_item[DD_WARPS];
     __shared__ int wcnt[DD_WARPS * DD_K];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     {
-        const int n = a.counters[CNT_COUNT + CLS_DD_CTA];
-        const int b = a.counters[CNT_BEGIN + CLS_DD_CTA];
+        const int n = a.counters[CNT_COUNT + C_CTA];
+        const int b = a.counters[CNT_BEGIN + C_CTA];
         for (;;) {
             __syncthreads();
-            if (threadIdx.x == 0) s_item[0] = atomicAdd(a.counters + CNT_HEAD + CLS_DD_CTA, 1);
+            if (threadIdx.x == 0) s_item[0] = atomicAdd(a.counters + CNT_HEAD + C_CTA, 1);
             __syncthreads();
             const int item = s_item[0];
             if (item >= n) break;
@@ -495,18 +513,22 @@ __global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupA
             int E = pow2_at_least(2 * T);
             if (E > DD_CTA_E) E = DD_CTA_E;
 #define F2_DD_CTA(W) dedup_ctx<DD_WARPS, W>(s, a, c, smem, E, wcnt)
-            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_CTA)
+            if constexpr (WX) {
+                F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_CTA)
+            } else {
+                F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_CTA)
+            }
 #undef F2_DD_CTA
         }
     }
     {
         const int q = warp / 4;
-        const int n = a.counters[CNT_COUNT + CLS_DD_QUAD];
-        const int b = a.counters[CNT_BEGIN + CLS_DD_QUAD];
+        const int n = a.counters[CNT_COUNT + C_QUAD];
+        const int b = a.counters[CNT_BEGIN + C_QUAD];
         uint32_t* region = smem + q * 4 * DD_WARP_REGION;
         for (;;) {
             dd_sync<4>();
-            if ((warp & 3) == 0 && lane == 0) s_item[q] = atomicAdd(a.counters + CNT_HEAD + CLS_DD_QUAD, 1);
+            if ((warp & 3) == 0 && lane == 0) s_item[q] = atomicAdd(a.counters + CNT_HEAD + C_QUAD, 1);
             dd_sync<4>();
             const int item = s_item[q];
             if (item >= n) break;
@@ -515,24 +537,32 @@ __global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupA
             int E = pow2_at_least(2 * T);
             if (E > DD_QUAD_E) E = DD_QUAD_E;
 #define F2_DD_QUAD(W) dedup_ctx<4, W>(s, a, c, region, E, wcnt + q * 4 * DD_K)
-            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_QUAD)
+            if constexpr (WX) {
+                F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_QUAD)
+            } else {
+                F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_QUAD)
+            }
 #undef F2_DD_QUAD
         }
     }
     {
-        const int n = a.counters[CNT_COUNT + CLS_DD_WARP];
-        const int b = a.counters[CNT_BEGIN + CLS_DD_WARP];
+        const int n = a.counters[CNT_COUNT + C_WARP];
+        const int b = a.counters[CNT_BEGIN + C_WARP];
         uint32_t* region = smem + warp * DD_WARP_REGION;
         for (;;) {
             int item = 0;
-            if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + CLS_DD_WARP, 1);
+            if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + C_WARP, 1);
             item = __shfl_sync(FULL, item, 0);
             if (item >= n) break;
             const int c = a.queue[b + item];
             const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
             const int E = pow2_at_least(2 * T);
 #define F2_DD_WARP(W) dedup_ctx<1, W>(s, a, c, region, E, nullptr)
-            F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_WARP)
+            if constexpr (WX) {
+                F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_WARP)
+            } else {
+                F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_WARP)
+            }
 #undef F2_DD_WARP
         }
     }
@@ -707,30 +737,33 @@ __device__ int insert_block(uint32_t (&xr)[WD], uint4& yr, uint32_t cand, uint32
     return __popc(newp);
 }
 
+// The stored basis moves between global and shared memory by its pivot rows
+// only: an empty slot is zero in the store and never read in shared memory
+// (every read of S selects a pivot), and a slot that became a pivot stays one.
 template <int WD>
-__device__ void basis_to_smem(const StoreDev& s, const CtxDesc& cd, uint32_t* S, int t, int nt)
+__device__ void basis_to_smem(const StoreDev& s, const CtxDesc& cd, uint32_t* S, const uint32_t* Ps, int t, int nt)
 {
     constexpr int RS = row_stride(WD);
     for (int k = t; k < cd.d; k += nt) {
-        *reinterpret_cast<uint4*>(S + k * RS) = s.bz[cd.slot_off + k];
-        for (int v = cd.wd; v < RS - 4; ++v) S[k * RS + 4 + v] = 0;
-    }
-    const int words = cd.d * cd.wd;
-    for (int idx = t; idx < words; idx += nt) {
-        const int k = idx / cd.wd, v = idx - k * cd.wd;
-        S[k * RS + 4 + v] = s.bx[cd.xw_off + idx];
+        if (!((Ps[k >> 5] >> (k & 31)) & 1u)) continue;
+        uint32_t* row = S + k * RS;
+        *reinterpret_cast<uint4*>(row) = s.bz[cd.slot_off + k];
+        const uint32_t* src = s.bx + cd.xw_off + (int64_t)k * cd.wd;
+        for (int v = 0; v < RS - 4; ++v) row[4 + v] = (v < cd.wd) ? src[v] : 0u;
     }
 }
 
 template <int WD>
-__device__ void basis_from_smem(const StoreDev& s, const CtxDesc& cd, const uint32_t* S, int t, int nt)
+__device__ void basis_from_smem(const StoreDev& s, const CtxDesc& cd, const uint32_t* S, const uint32_t* Ps, int t,
+                                int nt)
 {
     constexpr int RS = row_stride(WD);
-    for (int k = t; k < cd.d; k += nt) s.bz[cd.slot_off + k] = *reinterpret_cast<const uint4*>(S + k * RS);
-    const int words = cd.d * cd.wd;
-    for (int idx = t; idx < words; idx += nt) {
-        const int k = idx / cd.wd, v = idx - k * cd.wd;
-        s.bx[cd.xw_off + idx] = S[k * RS + 4 + v];
+    for (int k = t; k < cd.d; k += nt) {
+        if (!((Ps[k >> 5] >> (k & 31)) & 1u)) continue;
+        const uint32_t* row = S + k * RS;
+        s.bz[cd.slot_off + k] = *reinterpret_cast<const uint4*>(row);
+        uint32_t* dst = s.bx + cd.xw_off + (int64_t)k * cd.wd;
+        for (int v = 0; v < cd.wd; ++v) dst[v] = row[4 + v];
     }
 }
 
@@ -754,19 +787,6 @@ __device__ __forceinline__ void commit_stats(const StoreDev& s, int c, long long
 
 // ------------------------------------------------------------------ pass 2
 
-// Context c's basis into shared memory (a context of rank 0 has an all-zero
-// stored basis, so it is cleared instead of read).
-template <int WD>
-__device__ void basis_in(const StoreDev& s, const CtxDesc& cd, uint32_t* S, int t, int nt, bool empty)
-{
-    constexpr int RS = row_stride(WD);
-    if (empty) {
-        for (int w = t; w < cd.d * RS; w += nt) S[w] = 0u;
-        return;
-    }
-    basis_to_smem<WD>(s, cd, S, t, nt);
-}
-
 // One group (a warp, or the whole CTA) streams the representatives of
 // context c through its basis.
 template <int WD, bool CTA>
@@ -787,7 +807,6 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     long long* first_s = reinterpret_cast<long long*>(ctl + CTL_FIRST);
     uint32_t* S = region + CTL_WORDS;
     const int rank0 = s.rank[c];
-    basis_in<WD>(s, cd, S, t, nt, rank0 == 0);
     if (t < 48) {
         Ps[t] = (t < cd.wd && rank0 != 0) ? s.pivot[cd.pw_off + t] : 0u;
         NPR[t] = 0u;
@@ -798,6 +817,10 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
         *first_s = LLONG_MAX;
     }
     group_sync<CTA>();
+    if (rank0 != 0) {
+        basis_to_smem<WD>(s, cd, S, Ps, t, nt);
+        group_sync<CTA>();
+    }
     uint32_t P[WD];
 #pragma unroll
     for (int v = 0; v < WD; ++v) P[v] = Ps[v];
@@ -904,7 +927,7 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     }
     group_sync<CTA>();
     if (t < cd.wd) s.pivot[cd.pw_off + t] = Ps[t];
-    basis_from_smem<WD>(s, cd, S, t, nt);
+    basis_from_smem<WD>(s, cd, S, Ps, t, nt);
     if (t == 0) {
         s.rank[c] = *rank_s;
         commit_stats(s, c, *first_s, *cnt_s);
@@ -1044,7 +1067,7 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
             if (p.mode == 0 && p.rep_count) {
                 // wide rows are not deduplicated; rows of a full-rank context
                 // are checked one by one (verify_full_kernel)
-                if (R > 0 && (cd.xw > DD_XW || s.rank[c] == cd.d)) {
+                if (R > 0 && (cd.xw > DD_XW_WIDE || s.rank[c] == cd.d)) {
                     p.rep_count[c] = (int32_t)(-(R + 2));
                     R = 0;
                 } else {
@@ -1058,6 +1081,7 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
             unsigned long long work;
             if (p.mode == 0) {
                 cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : (R <= DD_QUAD_MAX_ROWS ? CLS_DD_QUAD : CLS_DD_CTA);
+                if (cd.xw > DD_XW) cls += CLS_DDW_CTA - CLS_DD_CTA;  // the 10..16-word instance
                 work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
             } else {
                 const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
@@ -1544,11 +1568,18 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         da.rep_count = st->rep_count;
         da.queue = st->queue;
         da.counters = st->counters;
-        e = cudaFuncSetAttribute(dedup_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
+        e = cudaFuncSetAttribute(dedup_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
         if (e != cudaSuccess) return f2_cuda_status(e);
-        dedup_kernel<<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+        dedup_kernel<false><<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
         e = cudaGetLastError();
         if (e != cudaSuccess) return f2_cuda_status(e);
+        if (st->max_xw > DD_XW) {  // some context has feature rows of 10..16 words
+            e = cudaFuncSetAttribute(dedup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
+            if (e != cudaSuccess) return f2_cuda_status(e);
+            dedup_kernel<true><<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return f2_cuda_status(e);
+        }
     }
     LearnArgs la;
     la.row_off = row_off;

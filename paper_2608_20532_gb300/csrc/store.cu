@@ -109,6 +109,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
         s->xw_off[(size_t)c + 1] = cd.xw_off + (int64_t)cd.d * cd.wd;
         s->pw_off[(size_t)c + 1] = cd.pw_off + cd.wd;
         if (cd.wd > s->max_wd) s->max_wd = cd.wd;
+        if (cd.xw > s->max_xw) s->max_xw = cd.xw;
         if (cd.d > s->max_d) s->max_d = cd.d;
         if (cd.wd > NARROW_WD) s->n_wide++;
     }

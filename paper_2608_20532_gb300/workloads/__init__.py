@@ -344,3 +344,95 @@ def onehot_offset(layout: int) -> int:
 def standard(cfg_id: int, **kw) -> Workload:
     """Configuration cfg_id at full size with its standard seed."""
     return generate(CONFIGS[cfg_id], seed_for(cfg_id), name=f"config{cfg_id}", **kw)
+
+
+# Parsed-value workload with the paper's exact-context rank statistics (input
+# synthesis only).  A context's observations carry k parsed int64 values;
+# phi(x) = [1 || bits64(v_0) || ... || bits64(v_{k-1})] (Sec. 2.1), so the
+# k values of a row, little-endian, are its n = 64k feature bits: x below is
+# the int64 values' memory seen as uint32 words.  Per context the evidence
+# rank r (of the [1 || x] rows) is log-normal with median 3 and 95th
+# percentile 21 (the SM107 statistics of Sec. 4), rows are ~200 per rank
+# (the ~200x compaction of the corpora), and x = offset XOR a random subset
+# of r - 1 sparse generators that flip low-order, mid-order or sign bits of
+# one value (register-, immediate- and sign-like fields).  y is a planted
+# affine map of x; a few contexts get one duplicate x with a flipped y bit.
+PARSED_LOWRANK = dict(num_ctx=10000, k_min=2, k_max=8, rank_median=3.0, rank_p95=21.0, rows_per_rank=200,
+                      rows_max=1 << 16, density=0.05, n_contra=20)
+
+
+def parsed_lowrank(seed: int = 20260006, **over) -> Workload:
+    p = dict(PARSED_LOWRANK, **over)
+    rng = np.random.default_rng(seed)
+    C = int(p["num_ctx"])
+    k = rng.integers(int(p["k_min"]), int(p["k_max"]) + 1, C)
+    n_bits = (64 * k).astype(np.int32)
+    sigma = np.log(p["rank_p95"] / p["rank_median"]) / 1.6449
+    r = np.rint(np.exp(rng.normal(np.log(p["rank_median"]), sigma, C))).astype(np.int64)
+    r = np.clip(r, 1, 64)
+    T = np.rint(r * p["rows_per_rank"] * np.exp(rng.normal(0.0, 0.5, C))).astype(np.int64)
+    T = np.clip(T, np.maximum(r, 2), int(p["rows_max"]))
+    contra_ctx = rng.choice(C, size=min(C, int(p["n_contra"])), replace=False)
+    W = (n_bits.astype(np.int64) + 31) // 32  # = 2k
+    row_off = np.zeros(C + 1, np.int64)
+    row_off[1:] = np.cumsum(T)
+    x_off = np.zeros(C, np.int64)
+    x_off[1:] = np.cumsum(T * W)[:-1]
+    R = int(T.sum())
+    x64 = np.zeros(int((T * k).sum()), np.int64)
+    y = np.zeros((R, 4), np.uint32)
+    a_off = np.zeros(C, np.int64)
+    a_off[1:] = np.cumsum(n_bits.astype(np.int64))[:-1]
+    A = np.zeros((int(n_bits.sum()), 4), np.uint32)
+    b = np.zeros((C, 4), np.uint32)
+    contra_pos = np.full(C, -1, np.int64)
+    contra_bit = np.full(C, -1, np.int32)
+    is_contra = np.zeros(C, bool)
+    is_contra[contra_ctx] = True
+    for c in range(C):
+        kc, n, Tc, rc = int(k[c]), int(n_bits[c]), int(T[c]), int(r[c])
+        # planted map: column j of A is the word of feature bit j
+        Ac = (rng.random((n, 128)) < p["density"])
+        Aw = np.packbits(Ac, axis=1, bitorder="little").view(np.uint32).reshape(n, 4)
+        bc = rng.integers(0, 2 ** 32, size=4, dtype=np.uint64).astype(np.uint32)
+        A[a_off[c]:a_off[c] + n] = Aw
+        b[c] = bc
+        # offset values (small, sometimes negative) and sparse generators
+        off = rng.integers(0, 256, kc).astype(np.int64)
+        off[rng.random(kc) < 0.1] *= -1
+        gens = np.zeros((max(rc - 1, 0), kc), np.int64)
+        for j in range(rc - 1):
+            i = rng.integers(kc)
+            u = rng.random()
+            bit = int(rng.integers(8)) if u < 0.6 else (int(rng.integers(8, 32)) if u < 0.95 else 63)
+            gens[j, i] = np.int64(1) << np.int64(bit) if bit < 63 else np.int64(-(1 << 63))
+        sel = rng.random((Tc, max(rc - 1, 0))) < 0.5
+        xv = np.tile(off, (Tc, 1))
+        for j in range(rc - 1):
+            xv[sel[:, j]] ^= gens[j]
+        # y = b XOR A x, evaluated through the generators (x is affine in sel)
+        def word(vals):
+            bits = np.unpackbits(vals.astype("<i8").view(np.uint8), bitorder="little")[:n].astype(bool)
+            return np.bitwise_xor.reduce(Aw[bits], axis=0) if bits.any() else np.zeros(4, np.uint32)
+        y_off = bc ^ word(off)
+        yc = np.tile(y_off, (Tc, 1))
+        for j in range(rc - 1):
+            yc[sel[:, j]] ^= word(gens[j])
+        if is_contra[c] and Tc > 1:
+            # a later copy of an earlier row's x with one flipped word bit
+            pos = int(rng.integers(1, Tc))
+            src = int(rng.integers(0, pos))
+            xv[pos] = xv[src]
+            yc[pos] = yc[src]
+            bit = int(rng.integers(128))
+            yc[pos, bit // 32] ^= np.uint32(1 << (bit % 32))
+            contra_pos[c] = pos
+            contra_bit[c] = bit
+        x64[x_off[c] // 2: x_off[c] // 2 + Tc * kc] = xv.reshape(-1)
+        y[row_off[c]:row_off[c + 1]] = yc
+    x = x64.view(np.uint32)
+    zeros = np.zeros(C, np.int64)
+    return Workload(name="parsed-lowrank", params=p, seed=seed, n_bits=n_bits, rows=T, fresh=r, dups=T - r,
+                    contra=is_contra.astype(np.uint8), two_stream=np.zeros(C, np.uint8), row_off=row_off,
+                    x_off=x_off, x=x, y=y, a_off=a_off, A=A, b=b, contra_pos=contra_pos, contra_bit=contra_bit,
+                    batches=[(row_off, x_off)], queries=None)

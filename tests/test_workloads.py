@@ -81,3 +81,27 @@ def test_zipf_queries():
     top = np.sort(counts)[::-1]
     assert top[0] > 10 * np.median(counts[counts > 0])  # heavy head
     assert abs((1 - q.expect_in.mean()) - 0.05) < 0.01
+
+
+def test_parsed_lowrank_layout_and_map():
+    """Parsed-value rows: x is the k int64 values' little-endian memory
+    (feature bit 64i + b = bit b of v_i, Sec. 2.1); y follows the planted
+    affine map except the one flipped duplicate of a contradiction context."""
+    wl = wlmod.parsed_lowrank(num_ctx=60, seed=3, rows_per_rank=20)
+    assert (wl.n_bits % 64 == 0).all() and wl.n_bits.min() >= 128 and wl.n_bits.max() <= 512
+    for c in range(wl.num_ctx):
+        xs, ys = wl.ctx_rows(c)
+        k = int(wl.n_bits[c]) // 64
+        vals = np.ascontiguousarray(xs).view(np.int64)
+        assert vals.shape == (int(wl.rows[c]), k)
+        n = int(wl.n_bits[c])
+        a0 = int(wl.a_off[c])
+        for i in range(0, len(xs), 7):
+            acc = wl.b[c].copy()
+            for j in range(n):
+                if (int(vals[i, j // 64]) >> (j % 64)) & 1:
+                    acc ^= wl.A[a0 + j]
+            flips = int(np.unpackbits((acc ^ ys[i]).view(np.uint8)).sum())
+            assert flips == (1 if i == wl.contra_pos[c] else 0)
+        # at most 2^(r-1) distinct x (an affine subspace of dimension r - 1)
+        assert len({bytes(r) for r in xs}) <= 2 ** (int(wl.fresh[c]) - 1)
