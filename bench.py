@@ -370,6 +370,31 @@ def run_ours(args):
                     "kernel": "epilogue_kernel (f2_encode_epilogue)"}
         del y_epi, state_t, sched_t
 
+    # ---- map pooling (Sec. 3): the exact contexts of each (f, m) group of the
+    # parsed-value workload merged into one store; the call synchronizes, so
+    # it is timed on the host clock, after the step
+    pooling = None
+    gs = int(wl.params.get("group_size", 0) or 0)
+    if gs > 0:
+        group_of = (np.arange(wl.num_ctx) // gs).astype(np.int32)
+        G = int(group_of[-1]) + 1
+        for _ in range(2):
+            store.merge(group_of, G)[0].close()
+        torch.cuda.synchronize()
+        t_m = time.perf_counter()
+        for _ in range(K):
+            merged, _ok = store.merge(group_of, G)
+            if _ < K - 1:
+                merged.close()
+        m_ms = (time.perf_counter() - t_m) * 1e3 / K
+        mb = merged.basis()
+        torch.cuda.synchronize()
+        pooling = {"ms": m_ms, "groups": G, "group_size": gs,
+                   "merged_rows": int(binding.to_numpy(b["rank"]).astype(np.int64).sum()),
+                   "shared_maps": int((binding.to_numpy(mb["contra"]) == 0).sum()),
+                   "call": "f2_merge_bases (merge_gather_kernel + learn kernels; host clock)"}
+        merged.close()
+
     # ---- e2e through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -504,6 +529,8 @@ def run_ours(args):
     if epilogue is not None:
         epilogue["frac_of_measured_hbm"] = epilogue["achieved_gbs"] / peaks["hbm_gbs"]
         result["encode_epilogue"] = epilogue
+    if pooling is not None:
+        result["map_pooling"] = pooling
     if e2e is not None:
         result["e2e"] = e2e
     if world == 1 and not args.no_cpu_baseline:

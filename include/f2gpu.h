@@ -177,6 +177,28 @@ int f2_encode_batched(const f2_store* store, int64_t Q, const int32_t* ctx_id_de
                       uint8_t* in_span_dev, f2_stream_t stream);
 
 /*
+ * Map pooling (Sec. 3: the bases of an (f, m) group are combined and
+ * eliminated together; one shared map if the equations are consistent and
+ * the output masks match, else separate maps).  group_of_host[c] in
+ * [0, num_groups) puts source context c in a group (-1: left out); every
+ * group needs at least one member and all members of a group the same d.
+ * *out receives a new store with F2_FLAG_RAW_FEATURES and one context per
+ * group of width d (its feature rows are phi-space vectors, index 0 = the
+ * constant): the members' basis rows, members in context order and pivots in
+ * increasing order, learned as one stream.  Its basis is the reduced echelon
+ * form of the union of the members' spans; its contradiction flag marks
+ * inconsistent equations (first_contra / n_contra count merged rows).
+ * out_mask_host (uint32[4*num_ctx], the learned output bits of each context;
+ * NULL: all equal) and mask_ok_host (uint8[num_groups], may be NULL): 1 where
+ * all members' masks are equal.  A group shares one map iff mask_ok and not
+ * contra.  The call synchronizes `stream`; destroy *out with f2_destroy.
+ * Errors: F2_ERR_INVALID_ARG, F2_ERR_CTX_RANGE (group id out of range),
+ * F2_ERR_NBITS (members of different widths), F2_ERR_OOM, F2_ERR_CUDA.
+ */
+int f2_merge_bases(const f2_store* src, int32_t num_groups, const int32_t* group_of_host,
+                   const uint32_t* out_mask_host, f2_store** out, uint8_t* mask_ok_host, f2_stream_t stream);
+
+/*
  * Encode epilogue (Appendix C, Eq. hmma-full-word; Appendix D): turns the
  * learned words of accepted queries into full instruction words, in place.
  * Scheduler control is kept outside the learned bits and merged at bits

@@ -96,6 +96,17 @@ class Basis:
         return [self.rows[k][1] if k in self.rows else 0 for k in range(self.d)]
 
 
+def merge_bases(d: int, bases: List["Basis"]) -> "Basis":
+    """Map pooling (Sec. 3): the bases of a group eliminated together, members
+    in order, each member's rows in increasing pivot order.  The result spans
+    the union of the members' spans; a contradiction means the members'
+    equations admit no single map."""
+    rows = []
+    for B in bases:
+        rows += [B.rows[k] for k in sorted(B.rows)]
+    return learn_rows(d, rows)
+
+
 SCHED_SHIFT = 105  # Appendix C: scheduler control occupies bits 105..121
 
 

@@ -39,7 +39,7 @@ EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
     "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3", "f2_learn_batched_noalloc",
-    "f2_encode_epilogue",
+    "f2_encode_epilogue", "f2_merge_bases",
 )
 
 _lib = None
@@ -78,6 +78,7 @@ def load_library(path: Optional[str] = None):
         "f2_solve_affine": ([P, P, P], ctypes.c_int),
         "f2_encode_batched": ([P, i64, P, P, i32, P, P, P], ctypes.c_int),
         "f2_encode_epilogue": ([P, i64, P, P, P, P, P, P, P], ctypes.c_int),
+        "f2_merge_bases": ([P, i32, P, P, ctypes.POINTER(P), P, P], ctypes.c_int),
         "f2_device_status": ([P, ctypes.POINTER(ctypes.c_int), P], ctypes.c_int),
         "f2_store_export": ([P, P, ctypes.POINTER(ctypes.c_size_t), P], ctypes.c_int),
         "f2_store_import": ([P, P, ctypes.c_size_t, P], ctypes.c_int),
@@ -124,16 +125,19 @@ def _dptr(t: Optional[torch.Tensor]):
 class Store:
     """A set of encoding contexts and their learned reduced bases on one GPU."""
 
-    def __init__(self, n_bits, raw: bool = False, device=None, stream=None):
+    def __init__(self, n_bits, raw: bool = False, device=None, stream=None, _handle=None):
         self._lib = load_library()
         nb = np.ascontiguousarray(np.asarray(n_bits, dtype=np.int32))
         self.n_bits = nb
         self.raw = bool(raw)
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
-        h = ctypes.c_void_p()
-        with torch.cuda.device(self.device):
-            _check(self._lib.f2_create(ctypes.byref(h), int(nb.shape[0]), nb.ctypes.data,
-                                       F2_FLAG_RAW_FEATURES if raw else 0, _stream(stream)), "f2_create")
+        if _handle is None:
+            h = ctypes.c_void_p()
+            with torch.cuda.device(self.device):
+                _check(self._lib.f2_create(ctypes.byref(h), int(nb.shape[0]), nb.ctypes.data,
+                                           F2_FLAG_RAW_FEATURES if raw else 0, _stream(stream)), "f2_create")
+        else:  # a store the library created (f2_merge_bases)
+            h = _handle
         self._h = h
         n = int(nb.shape[0]) + 1
         self.slot_off = np.zeros(n, np.int64)
@@ -220,6 +224,24 @@ class Store:
                                             _dptr(opaque_mask) if opaque_mask is not None else None,
                                             _dptr(y), _stream(stream)), "f2_encode_epilogue")
         return y
+
+    def merge(self, group_of, num_groups: int, out_mask=None, stream=None):
+        """Map pooling: the bases of each group of contexts eliminated together
+        (f2_merge_bases).  Returns (store with one raw-feature context per
+        group, mask_ok uint8[num_groups])."""
+        g = np.ascontiguousarray(np.asarray(group_of, dtype=np.int32))
+        m = None if out_mask is None else np.ascontiguousarray(np.asarray(out_mask, dtype=np.uint32))
+        ok = np.zeros(max(int(num_groups), 1), np.uint8)
+        h = ctypes.c_void_p()
+        with torch.cuda.device(self.device):
+            _check(self._lib.f2_merge_bases(self._h, int(num_groups), g.ctypes.data,
+                                            m.ctypes.data if m is not None else None, ctypes.byref(h),
+                                            ok.ctypes.data, _stream(stream)), "f2_merge_bases")
+        d = np.zeros(int(num_groups), np.int32)
+        for c in range(len(g)):
+            if g[c] >= 0:
+                d[g[c]] = self.n_bits[c] + (0 if self.raw else 1)
+        return Store(d, raw=True, device=self.device, _handle=h), ok[:int(num_groups)]
 
     def device_status(self, stream=None) -> int:
         v = ctypes.c_int(0)

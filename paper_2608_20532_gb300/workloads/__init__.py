@@ -357,15 +357,19 @@ def standard(cfg_id: int, **kw) -> Workload:
 # of r - 1 sparse generators that flip low-order, mid-order or sign bits of
 # one value (register-, immediate- and sign-like fields).  y is a planted
 # affine map of x; a few contexts get one duplicate x with a flipped y bit.
+# Consecutive contexts in groups of group_size share k and the planted map:
+# the exact contexts of one (f, m) group, which differ in their operand
+# signature (and so in their input subspace) but not in the map (Sec. 3).
 PARSED_LOWRANK = dict(num_ctx=10000, k_min=2, k_max=8, rank_median=3.0, rank_p95=21.0, rows_per_rank=200,
-                      rows_max=1 << 16, density=0.05, n_contra=20)
+                      rows_max=1 << 16, density=0.05, n_contra=20, group_size=8)
 
 
 def parsed_lowrank(seed: int = 20260006, **over) -> Workload:
     p = dict(PARSED_LOWRANK, **over)
     rng = np.random.default_rng(seed)
     C = int(p["num_ctx"])
-    k = rng.integers(int(p["k_min"]), int(p["k_max"]) + 1, C)
+    gs = max(1, int(p["group_size"]))
+    k = np.repeat(rng.integers(int(p["k_min"]), int(p["k_max"]) + 1, (C + gs - 1) // gs), gs)[:C]
     n_bits = (64 * k).astype(np.int32)
     sigma = np.log(p["rank_p95"] / p["rank_median"]) / 1.6449
     r = np.rint(np.exp(rng.normal(np.log(p["rank_median"]), sigma, C))).astype(np.int64)
@@ -391,10 +395,10 @@ def parsed_lowrank(seed: int = 20260006, **over) -> Workload:
     is_contra[contra_ctx] = True
     for c in range(C):
         kc, n, Tc, rc = int(k[c]), int(n_bits[c]), int(T[c]), int(r[c])
-        # planted map: column j of A is the word of feature bit j
-        Ac = (rng.random((n, 128)) < p["density"])
-        Aw = np.packbits(Ac, axis=1, bitorder="little").view(np.uint32).reshape(n, 4)
-        bc = rng.integers(0, 2 ** 32, size=4, dtype=np.uint64).astype(np.uint32)
+        if c % gs == 0:  # planted map of the group: column j of A is the word of feature bit j
+            Ac = (rng.random((n, 128)) < p["density"])
+            Aw = np.packbits(Ac, axis=1, bitorder="little").view(np.uint32).reshape(n, 4)
+            bc = rng.integers(0, 2 ** 32, size=4, dtype=np.uint64).astype(np.uint32)
         A[a_off[c]:a_off[c] + n] = Aw
         b[c] = bc
         # offset values (small, sometimes negative) and sparse generators
