@@ -177,6 +177,41 @@ int f2_encode_batched(const f2_store* store, int64_t Q, const int32_t* ctx_id_de
                       uint8_t* in_span_dev, f2_stream_t stream);
 
 /*
+ * Learning from host memory (Sec. 2.2, as f2_learn_batched): the same CSR
+ * batch, but row_off_host, x_host, x_off_host and y_host are host arrays
+ * (page-locked memory lets the copies overlap the kernels; pageable memory
+ * works, with the copies serialised).  The batch is validated on the host
+ * (F2_ERR_INVALID_ARG for decreasing offsets, offsets outside the arrays)
+ * and cut into chunks of whole contexts of about F2_OPT_HOST_CHUNK_BYTES of
+ * rows; a private copy stream moves chunk j + 1 into a device double buffer
+ * while `stream` learns chunk j.  The resulting state equals one
+ * f2_learn_batched call on the same batch (contexts are independent).  The
+ * host arrays are read asynchronously: keep them unchanged until `stream`
+ * has passed the call.  Device scratch: two chunk buffers and the rebased
+ * offsets (16 bytes per context), grown on demand (the call then
+ * synchronizes `stream`); kept by the store until f2_destroy.
+ */
+int f2_learn_host(f2_store* store, const int64_t* row_off_host, const uint32_t* x_host,
+                  const int64_t* x_off_host, const uint32_t* y_host, int64_t total_rows,
+                  int64_t total_x_words, f2_stream_t stream);
+
+/*
+ * Encoding from and to host memory (Sec. 2.3, as f2_encode_batched):
+ * ctx_id_host int32[Q], x_host uint32[Q * x_stride_words], y_out_host
+ * uint32[4 * Q], in_span_host uint8[Q] are host arrays (page-locked for
+ * overlap).  Queries go in chunks of at most F2_OPT_HOST_CHUNK_BYTES (and at
+ * least four chunks of at least 65,536 queries when Q allows): chunk
+ * j + 1 is copied in on a private stream while `stream` encodes chunk j and
+ * a second private stream copies the words of chunk j - 1 out.  Results are
+ * those of f2_encode_batched; device errors are recorded in the store's
+ * status word as there.  The outputs are written asynchronously: they are on
+ * the host once `stream` has passed the call.  Errors: F2_ERR_INVALID_ARG
+ * (Q < 0, NULL pointers, x_stride_words < 1), F2_ERR_OOM, F2_ERR_CUDA.
+ */
+int f2_encode_host(const f2_store* store, int64_t Q, const int32_t* ctx_id_host, const uint32_t* x_host,
+                   int32_t x_stride_words, uint32_t* y_out_host, uint8_t* in_span_host, f2_stream_t stream);
+
+/*
  * Map pooling (Sec. 3: the bases of an (f, m) group are combined and
  * eliminated together; one shared map if the equations are consistent and
  * the output masks match, else separate maps).  group_of_host[c] in
@@ -244,9 +279,11 @@ enum f2_option {
     F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context */
     F2_OPT_DEDUP = 4,            /* 1 (default): eliminate only the first occurrence of each distinct
                                     row and classify its repeats with it; 0: eliminate every row */
-    F2_OPT_ENCODE_TABLE_MIN = 5  /* shortest run of queries of one context (within a block of 2,048
+    F2_OPT_ENCODE_TABLE_MIN = 5, /* shortest run of queries of one context (within a block of 2,048
                                     grouped queries) encoded with a lookup table of its basis; default
                                     32, at least 16; a value above 2,048 disables the tables */
+    F2_OPT_HOST_CHUNK_BYTES = 6  /* bytes of rows (f2_learn_host) or of queries (f2_encode_host) per
+                                    copied chunk; default 512 MiB, at least 64 KiB */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

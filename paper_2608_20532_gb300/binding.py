@@ -33,13 +33,14 @@ F2_OPT_WARP_BASIS_BYTES = 2
 F2_OPT_WARP_WORK = 3
 F2_OPT_DEDUP = 4
 F2_OPT_ENCODE_TABLE_MIN = 5
+F2_OPT_HOST_CHUNK_BYTES = 6
 
 # every entry point of include/f2gpu.h
 EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
     "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3", "f2_learn_batched_noalloc",
-    "f2_encode_epilogue", "f2_merge_bases",
+    "f2_encode_epilogue", "f2_merge_bases", "f2_learn_host", "f2_encode_host",
 )
 
 _lib = None
@@ -77,6 +78,8 @@ def load_library(path: Optional[str] = None):
         "f2_get_basis": ([P] + [P] * 8 + [P], ctypes.c_int),
         "f2_solve_affine": ([P, P, P], ctypes.c_int),
         "f2_encode_batched": ([P, i64, P, P, i32, P, P, P], ctypes.c_int),
+        "f2_learn_host": ([P, P, P, P, P, i64, i64, P], ctypes.c_int),
+        "f2_encode_host": ([P, i64, P, P, i32, P, P, P], ctypes.c_int),
         "f2_encode_epilogue": ([P, i64, P, P, P, P, P, P, P], ctypes.c_int),
         "f2_merge_bases": ([P, i32, P, P, ctypes.POINTER(P), P, P], ctypes.c_int),
         "f2_device_status": ([P, ctypes.POINTER(ctypes.c_int), P], ctypes.c_int),
@@ -110,6 +113,23 @@ def _check(code: int, what: str):
 def _stream(stream=None) -> int:
     s = stream if stream is not None else torch.cuda.current_stream()
     return int(s.cuda_stream)
+
+
+def _hptr(a):
+    """Address of a host array (CPU tensor, ideally pinned, or numpy array)."""
+    if isinstance(a, torch.Tensor):
+        if a.is_cuda or not a.is_contiguous():
+            raise ValueError("expected a contiguous CPU tensor")
+        return a.data_ptr()
+    if isinstance(a, np.ndarray):
+        if not a.flags["C_CONTIGUOUS"]:
+            raise ValueError("expected a contiguous array")
+        return a.ctypes.data
+    raise TypeError("expected a CPU tensor or a numpy array")
+
+
+def _hsize(a) -> int:
+    return a.numel() if isinstance(a, torch.Tensor) else a.size
 
 
 def _dptr(t: Optional[torch.Tensor]):
@@ -148,8 +168,9 @@ class Store:
 
     def close(self):
         if getattr(self, "_h", None) and self._h.value:
-            self._lib.f2_destroy(self._h)
+            self._lib.f2_destroy(self._h)  # frees device memory: the device has synchronized
             self._h = ctypes.c_void_p()
+        self._held = []
 
     def __del__(self):
         try:
@@ -175,6 +196,36 @@ class Store:
         _check(self._lib.f2_learn_batched(self._h, _dptr(row_off), _dptr(x), _dptr(x_off), _dptr(y),
                                           int(total_rows), int(x.numel()), _stream(stream)),
                "f2_learn_batched")
+
+    def _hold(self, arrays, stream):
+        """Keep host arrays alive until `stream` has passed the call that reads or writes them."""
+        held = getattr(self, "_held", None)
+        if held is None:
+            held = self._held = []
+        held[:] = [(ev, refs) for ev, refs in held if not ev.query()]
+        ev = torch.cuda.Event()
+        ev.record(stream if stream is not None else torch.cuda.current_stream(self.device))
+        held.append((ev, tuple(arrays)))
+
+    def learn_host(self, row_off, x, x_off, y, stream=None):
+        """One batch from host memory (f2_learn_host): row_off int64[C+1], x 32-bit words,
+        x_off int64[C], y 32-bit words [R, 4]; pinned CPU tensors let copies overlap."""
+        with torch.cuda.device(self.device):
+            _check(self._lib.f2_learn_host(self._h, _hptr(row_off), _hptr(x), _hptr(x_off), _hptr(y),
+                                           int(_hsize(y) // 4), int(_hsize(x)), _stream(stream)),
+                   "f2_learn_host")
+            self._hold((row_off, x, x_off, y), stream)
+
+    def encode_host(self, ctx_id, x, y_out, in_span, stream=None):
+        """Queries in host memory (f2_encode_host): ctx_id int32[Q], x 32-bit words [Q, stride];
+        y_out 32-bit words [Q, 4] and in_span uint8[Q] are written once `stream` passes the call."""
+        Q = int(_hsize(ctx_id))
+        stride = int(x.shape[1]) if len(x.shape) == 2 else 1
+        with torch.cuda.device(self.device):
+            _check(self._lib.f2_encode_host(self._h, Q, _hptr(ctx_id), _hptr(x), stride, _hptr(y_out),
+                                            _hptr(in_span), _stream(stream)), "f2_encode_host")
+            self._hold((ctx_id, x, y_out, in_span), stream)
+        return y_out, in_span
 
     def basis(self, stream=None) -> dict:
         C = self.num_ctx

@@ -10,6 +10,8 @@
 
 namespace f2 {
 
+struct HostIO;  // copy streams, events and staging of the host-input entry points
+
 constexpr unsigned FULL = 0xffffffffu;
 constexpr int MAX_N = 1024;          // feature bits per context
 constexpr int MAX_D = MAX_N + 1;     // row width with the affine constant
@@ -50,6 +52,14 @@ enum Class {
 static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
 constexpr int SMALL_WD = 3;
 constexpr int PLAN_HIST_WORDS = 8192;  // key histogram of the plan kernels (>= number of keys)  // contexts of d <= 96 bits: fewer registers, twice the warps per SM
+
+// Shared-memory and kernel selection of the elimination launches: the widest
+// rows of each width class of a store.
+struct Widths {
+    int max_small_words = 0, max_narrow_words = 0, max_wide_d = 0;
+    int max_d = 0, max_xw = 0;  // over every context (any may reach full rank)
+    bool has_small = false, has_narrow = false, has_wide = false;
+};
 
 // Per-context descriptor (device copy built at store creation).
 struct CtxDesc {
@@ -106,6 +116,8 @@ struct f2_store {
     int64_t warp_basis_bytes;
     int64_t warp_work;
     int dedup;              // run the duplicate pass before elimination
+    f2::Widths widths;      // width classes of the contexts (computed on first use)
+    bool widths_ready;
     std::vector<int32_t> n_bits;
     std::vector<int64_t> slot_off, xw_off, pw_off;
     // device memory
@@ -144,6 +156,9 @@ struct f2_store {
     mutable int64_t enc_q_cap;
     mutable int enc_short_per_sm;           // resident CTAs of the per-warp encode kernel
     int enc_table_min;                      // shortest run encoded with a table
+    // host-input entry points (f2_learn_host, f2_encode_host)
+    f2::HostIO* hio;
+    int64_t host_chunk_bytes;               // bytes of rows (or queries) per copied chunk
 
     f2::StoreDev dev() const
     {
@@ -164,7 +179,10 @@ struct f2_store {
     }
 };
 
-// Host helpers (store.cu, encode.cu).
+constexpr int64_t DEFAULT_HOST_CHUNK_BYTES = int64_t(512) << 20;
+
+// Host helpers (store.cu, encode.cu, host_io.cu).
+void f2_host_io_free(f2_store* st);
 int f2_cuda_status(cudaError_t e);
 int f2_encode_table_min_default();
 int f2_encode_table_min_floor();

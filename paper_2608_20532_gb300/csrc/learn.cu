@@ -1384,11 +1384,6 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
 }
 
 // Which elimination kernels a store needs, and their widest bases.
-struct Widths {
-    int max_small_words = 0, max_narrow_words = 0, max_wide_d = 0;
-    int max_d = 0, max_xw = 0;  // over every context (any may reach full rank)
-    bool has_small = false, has_narrow = false, has_wide = false;
-};
 
 size_t narrow_smem(int max_narrow_words, int warp_region_words)
 {
@@ -1592,7 +1587,11 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     la.queue = st->queue;
     la.counters = st->counters;
     la.warp_region_words = (int)(st->warp_basis_bytes / 4);
-    const Widths wv = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
+    if (!st->widths_ready) {  // fixed by the widths: computed once per store
+        st->widths = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
+        st->widths_ready = true;
+    }
+    const Widths& wv = st->widths;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
                               wv, st->full_ctr, st->full_cnt, st->full_first, cs);

@@ -37,6 +37,7 @@ extern "C" const char* f2_status_string(int status)
 static void free_store(f2_store* s)
 {
     if (!s) return;
+    f2_host_io_free(s);
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
@@ -84,6 +85,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->warp_work = DEFAULT_WARP_WORK;
     s->dedup = 1;
     s->enc_table_min = f2_encode_table_min_default();
+    s->host_chunk_bytes = DEFAULT_HOST_CHUNK_BYTES;
     if (cudaGetDevice(&s->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
         delete s;
@@ -380,6 +382,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_ENCODE_TABLE_MIN:
         if (value < f2_encode_table_min_floor() || value > (int64_t(1) << 30)) return F2_ERR_INVALID_ARG;
         s->enc_table_min = (int)value;
+        return F2_OK;
+    case F2_OPT_HOST_CHUNK_BYTES:
+        if (value < (int64_t(1) << 16)) return F2_ERR_INVALID_ARG;
+        s->host_chunk_bytes = value;
         return F2_OK;
     default:
         return F2_ERR_INVALID_ARG;
