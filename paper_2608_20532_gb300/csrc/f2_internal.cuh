@@ -117,6 +117,10 @@ struct f2_store {
     int64_t warp_work;
     int dedup;              // run the duplicate pass before elimination
     f2::Widths widths;      // width classes of the contexts (computed on first use)
+    // second stream of the learn launches (kernels of independent width
+    // classes run side by side), its fork and join events; created on first use
+    cudaStream_t aux;
+    cudaEvent_t ev_fork, ev_join;
     bool widths_ready;
     std::vector<int32_t> n_bits;
     std::vector<int64_t> slot_off, xw_off, pw_off;

@@ -1392,12 +1392,39 @@ size_t narrow_smem(int max_narrow_words, int warp_region_words)
     return cta > warps ? cta : warps;
 }
 
+// A second stream for kernels that work on disjoint contexts: the first
+// such kernel goes to `aux` (forked from the caller's stream), the others to
+// the caller's stream, and join() makes the caller's stream wait for `aux`.
+struct Fork {
+    cudaStream_t cs, aux;
+    cudaEvent_t ev_fork, ev_join;
+    bool forked = false;
+    cudaError_t e = cudaSuccess;
+    cudaStream_t next(int kernels_left)
+    {
+        if (!aux || forked || kernels_left < 2) return cs;
+        e = cudaEventRecord(ev_fork, cs);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(aux, ev_fork, 0);
+        if (e != cudaSuccess) return cs;
+        forked = true;
+        return aux;
+    }
+    cudaError_t join()
+    {
+        if (!forked || e != cudaSuccess) return e;
+        forked = false;
+        e = cudaEventRecord(ev_join, aux);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_join, 0);
+        return e;
+    }
+};
+
 // Enqueue pass 2 (plan + kernels) for one batch.
 int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* row_off, const int64_t* x_off,
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
-                       unsigned long long* full_first, cudaStream_t cs)
+                       unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr)
 {
     // full_ctr: chunks claimed [C], chunks done [C], late start [C], late list [C], late count
     const int C = sd.num_ctx;
@@ -1427,34 +1454,47 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     int rc = launch_plan(sd, pa, num_sms, cs);
     if (rc != F2_OK) return rc;
     cudaError_t e;
-    auto narrow = [&](auto kernel, size_t smem) -> int {
+    auto narrow = [&](auto kernel, size_t smem, cudaStream_t ks) -> int {
         cudaError_t er = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         int per_sm = 0;
         er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, LEARN_WARPS * 32, smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         if (per_sm < 1) per_sm = 1;
-        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, cs>>>(sd, lx);
+        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, ks>>>(sd, lx);
         return f2_cuda_status(cudaGetLastError());
     };
-    if (wv.has_small) {
-        const size_t words = (size_t)LEARN_WARPS * SMALL_REGION_WORDS;
-        rc = narrow(elim_narrow_kernel<true>,
-                    4 * (words > (size_t)wv.max_small_words ? words : (size_t)wv.max_small_words));
-        if (rc != F2_OK) return rc;
-    }
-    if (wv.has_narrow) {
-        rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words));
-        if (rc != F2_OK) return rc;
-    }
+    // the three width classes hold disjoint contexts: with a second stream
+    // their kernels overlap (each fills the others' tails)
+    Fork solo{cs, nullptr, nullptr, nullptr};
+    Fork& f = fk ? *fk : solo;
+    int left = (int)wv.has_narrow + (int)wv.has_wide + (int)wv.has_small;
     if (wv.has_wide) {
         const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
         e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return f2_cuda_status(e);
-        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, cs>>>(sd, lx);
+        const cudaStream_t ks = f.next(left--);
+        if (f.e != cudaSuccess) return f2_cuda_status(f.e);
+        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, ks>>>(sd, lx);
         e = cudaGetLastError();
         if (e != cudaSuccess) return f2_cuda_status(e);
     }
+    if (wv.has_narrow) {
+        const cudaStream_t ks = f.next(left--);
+        if (f.e != cudaSuccess) return f2_cuda_status(f.e);
+        rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words), ks);
+        if (rc != F2_OK) return rc;
+    }
+    if (wv.has_small) {
+        const size_t words = (size_t)LEARN_WARPS * SMALL_REGION_WORDS;
+        const cudaStream_t ks = f.next(left--);
+        if (f.e != cudaSuccess) return f2_cuda_status(f.e);
+        rc = narrow(elim_narrow_kernel<true>,
+                    4 * (words > (size_t)wv.max_small_words ? words : (size_t)wv.max_small_words), ks);
+        if (rc != F2_OK) return rc;
+    }
+    e = f.join();
+    if (e != cudaSuccess) return f2_cuda_status(e);
     {  // full-rank contexts: at the start of the call (the plan decides on the
        // device which, if any) or reached during it (listed by the kernels above)
         e = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
@@ -1536,6 +1576,17 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         st->rep_capacity = total_rows;
     }
     const StoreDev sd = st->dev();
+    if (!st->aux) {  // on the store's device
+        int cur = -1;
+        e = cudaGetDevice(&cur);
+        if (e == cudaSuccess && cur != st->device) e = cudaSetDevice(st->device);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_fork, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_join, cudaEventDisableTiming);
+        if (cur >= 0 && cur != st->device) cudaSetDevice(cur);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
+    Fork fk{cs, st->aux, st->ev_fork, st->ev_join};
     if (dedup) {
         PlanArgs pa;
         pa.row_off = row_off;
@@ -1563,18 +1614,24 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         da.rep_count = st->rep_count;
         da.queue = st->queue;
         da.counters = st->counters;
+        // the two instances hold disjoint contexts: side by side when both run
+        const bool wide_rows = st->max_xw > DD_XW;  // some context has feature rows of 10..16 words
         e = cudaFuncSetAttribute(dedup_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
         if (e != cudaSuccess) return f2_cuda_status(e);
-        dedup_kernel<false><<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+        cudaStream_t ks = fk.next(wide_rows ? 2 : 1);
+        if (fk.e != cudaSuccess) return f2_cuda_status(fk.e);
+        dedup_kernel<false><<<st->num_sms, DD_THREADS, DD_SMEM, ks>>>(sd, da);
         e = cudaGetLastError();
         if (e != cudaSuccess) return f2_cuda_status(e);
-        if (st->max_xw > DD_XW) {  // some context has feature rows of 10..16 words
+        if (wide_rows) {
             e = cudaFuncSetAttribute(dedup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
             if (e != cudaSuccess) return f2_cuda_status(e);
             dedup_kernel<true><<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
             e = cudaGetLastError();
             if (e != cudaSuccess) return f2_cuda_status(e);
         }
+        e = fk.join();
+        if (e != cudaSuccess) return f2_cuda_status(e);
     }
     LearnArgs la;
     la.row_off = row_off;
@@ -1594,7 +1651,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     const Widths& wv = st->widths;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
-                              wv, st->full_ctr, st->full_cnt, st->full_first, cs);
+                              wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk);
 }
 
 // ---------------------------------------------------------------------------

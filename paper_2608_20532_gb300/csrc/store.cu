@@ -38,6 +38,9 @@ static void free_store(f2_store* s)
 {
     if (!s) return;
     f2_host_io_free(s);
+    if (s->aux) cudaStreamDestroy(s->aux);
+    if (s->ev_fork) cudaEventDestroy(s->ev_fork);
+    if (s->ev_join) cudaEventDestroy(s->ev_join);
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
