@@ -47,7 +47,8 @@ enum Class {
     CLS_DDW_CTA = 9,   // dedup of feature rows of 10..16 words (their own kernel)
     CLS_DDW_QUAD = 10,
     CLS_DDW_WARP = 11,
-    NUM_CLASSES = 12
+    CLS_WIDE_M = 12,   // elimination of rows of 10..17 words (a narrower instance of the wide kernel)
+    NUM_CLASSES = 13
 };
 static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
 constexpr int SMALL_WD = 3;
@@ -56,9 +57,9 @@ constexpr int PLAN_HIST_WORDS = 8192;  // key histogram of the plan kernels (>= 
 // Shared-memory and kernel selection of the elimination launches: the widest
 // rows of each width class of a store.
 struct Widths {
-    int max_small_words = 0, max_narrow_words = 0, max_wide_d = 0;
+    int max_small_words = 0, max_narrow_words = 0, max_wide_m_d = 0, max_wide_d = 0;
     int max_d = 0, max_xw = 0;  // over every context (any may reach full rank)
-    bool has_small = false, has_narrow = false, has_wide = false;
+    bool has_small = false, has_narrow = false, has_wide_m = false, has_wide = false;
 };
 
 // Per-context descriptor (device copy built at store creation).

@@ -995,21 +995,24 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
     }
 }
 
-constexpr int WIDE_WD = 33;
+constexpr int WIDE_WD = 33;    // widest row (d <= 1056)
+constexpr int WIDE_M_WD = 17;  // rows of 10..17 words (d <= 544): half the registers, two CTAs per SM
 
-__global__ void __launch_bounds__(WIDE_WARPS * 32) elim_wide_kernel(StoreDev s, LearnArgs a)
+// Wide elimination: every context by a whole CTA, rows of up to WDT words.
+template <int WDT, int CLS>
+__global__ void __launch_bounds__(WIDE_WARPS * 32, WDT <= WIDE_M_WD ? 2 : 1) elim_wide_kernel(StoreDev s, LearnArgs a)
 {
     extern __shared__ __align__(16) uint32_t smem[];
     __shared__ int s_item;
-    const int n = a.counters[CNT_COUNT + CLS_WIDE];
-    const int b = a.counters[CNT_BEGIN + CLS_WIDE];
+    const int n = a.counters[CNT_COUNT + CLS];
+    const int b = a.counters[CNT_BEGIN + CLS];
     for (;;) {
         __syncthreads();
-        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_WIDE, 1);
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS, 1);
         __syncthreads();
         const int item = s_item;
         if (item >= n) break;
-        elim_ctx<WIDE_WD, true>(s, a, a.queue[b + item], smem);
+        elim_ctx<WDT, true>(s, a, a.queue[b + item], smem);
     }
 }
 
@@ -1087,7 +1090,7 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
                 const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
                                    R * cd.d > p.warp_work;
                 if (s.rank[c] == cd.d) cls = CLS_FULL;
-                else if (cd.wd > NARROW_WD) cls = CLS_WIDE;
+                else if (cd.wd > NARROW_WD) cls = (cd.wd <= WIDE_M_WD) ? CLS_WIDE_M : CLS_WIDE;
                 else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
                 else cls = heavy ? CLS_CTA : CLS_WARP;
                 work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
@@ -1468,16 +1471,27 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     // their kernels overlap (each fills the others' tails)
     Fork solo{cs, nullptr, nullptr, nullptr};
     Fork& f = fk ? *fk : solo;
-    int left = (int)wv.has_narrow + (int)wv.has_wide + (int)wv.has_small;
-    if (wv.has_wide) {
-        const size_t smem = 4 * (size_t)elim_words(wv.max_wide_d, WIDE_WD);
-        e = cudaFuncSetAttribute(elim_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+    int left = (int)wv.has_narrow + (int)wv.has_wide + (int)wv.has_wide_m + (int)wv.has_small;
+    auto wide = [&](auto kernel, int max_d, int wdt) -> int {
+        const size_t smem = 4 * (size_t)elim_words(max_d, wdt);
+        cudaError_t er = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (er != cudaSuccess) return f2_cuda_status(er);
+        int per_sm = 0;
+        er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, WIDE_WARPS * 32, smem);
+        if (er != cudaSuccess) return f2_cuda_status(er);
+        if (per_sm < 1) per_sm = 1;
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
-        elim_wide_kernel<<<num_sms, WIDE_WARPS * 32, smem, ks>>>(sd, lx);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        kernel<<<num_sms * per_sm, WIDE_WARPS * 32, smem, ks>>>(sd, lx);
+        return f2_cuda_status(cudaGetLastError());
+    };
+    if (wv.has_wide) {
+        rc = wide(elim_wide_kernel<WIDE_WD, CLS_WIDE>, wv.max_wide_d, WIDE_WD);
+        if (rc != F2_OK) return rc;
+    }
+    if (wv.has_wide_m) {
+        rc = wide(elim_wide_kernel<WIDE_M_WD, CLS_WIDE_M>, wv.max_wide_m_d, WIDE_M_WD);
+        if (rc != F2_OK) return rc;
     }
     if (wv.has_narrow) {
         const cudaStream_t ks = f.next(left--);
@@ -1543,6 +1557,9 @@ Widths width_summary(const int32_t* n_bits, int32_t num_ctx, bool raw)
         } else if (wd <= NARROW_WD) {
             w.has_narrow = true;
             if (words > w.max_narrow_words) w.max_narrow_words = words;
+        } else if (wd <= WIDE_M_WD) {
+            w.has_wide_m = true;
+            if (d > w.max_wide_m_d) w.max_wide_m_d = d;
         } else {
             w.has_wide = true;
             if (d > w.max_wide_d) w.max_wide_d = d;
