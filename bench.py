@@ -585,26 +585,30 @@ def basis_bytes_touched(wl, store) -> int:
     return int((d * (16 + 4 * wd) + 4 * wd).sum())
 
 
-def kernel_source_hash() -> str:
+# the translation units of each library call's kernels
+KERNEL_SOURCES = {"f2_learn_batched": ("learn.cu", "f2_internal.cuh"),
+                  "f2_encode_batched": ("encode.cu", "f2_internal.cuh")}
+
+
+def kernel_source_hash(call: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_20532_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, f), "rb") as fh:
-                h.update(fh.read())
+    for f in KERNEL_SOURCES[call]:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def profile_traffic(kernel: str):
-    """DRAM bytes per launch from a committed ncu summary, if it was taken on
-    the current kernel sources (null otherwise)."""
+def profile_traffic(call: str):
+    """DRAM bytes per call from a committed ncu summary, if it was taken on
+    the current sources of that call's kernels (null otherwise)."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as f:
         d = json.load(f)
-    e = d.get(kernel)
-    if not e or e.get("source_hash") != kernel_source_hash():
+    e = d.get(call)
+    if not e or e.get("source_hash") != kernel_source_hash(call):
         return None
     return e.get("dram_bytes_per_launch")
 
