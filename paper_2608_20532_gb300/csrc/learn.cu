@@ -87,20 +87,23 @@ constexpr int CTL_WORDS = 176; // size of the control area (16-byte multiple)
 constexpr int FULL_THREADS = 1024;  // verify_full_kernel: one table shared by 32 warps
 constexpr int FULL_CHUNK = 2048;   // rows of a full-rank context claimed at a time
 
-// Pass 1: 16 warps per CTA, one CTA per SM.  A warp-owned context (at most
-// DD_WARP_MAX_ROWS rows) gets a table of next_pow2(2T) entries in a 12 KB
+// Pass 1: 16 warps per CTA, two CTAs per SM (64 registers a thread: the pass
+// is bound by dependent per-row chains, so warps hide latency better than
+// rows held in flight by one warp).  A warp-owned context (at most
+// DD_WARP_MAX_ROWS rows) gets a table of next_pow2(2T) entries in a 6 KB
 // region; a CTA-owned context a table of up to DD_CTA_E entries.  Entry =
 // (fingerprint, row index) plus a duplicate counter: 12 bytes.
 constexpr int DD_THREADS = 512;
 constexpr int DD_WARPS = DD_THREADS / 32;
-constexpr int DD_WARP_MAX_ROWS = 512;           // warp-owned up to this many rows
-constexpr int DD_QUAD_MAX_ROWS = 8192;          // 4-warp-owned up to this many rows
-constexpr int DD_WARP_E = 1024;
+constexpr int DD_CTAS_PER_SM = 2;
+constexpr int DD_WARP_MAX_ROWS = 256;           // warp-owned up to this many rows
+constexpr int DD_QUAD_MAX_ROWS = 4096;          // 4-warp-owned up to this many rows
+constexpr int DD_WARP_E = 512;
 constexpr int DD_WARP_REGION = 3 * DD_WARP_E;   // words
 constexpr int DD_QUAD_E = 4 * DD_WARP_E;
-constexpr int DD_CTA_E = 16384;
+constexpr int DD_CTA_E = 8192;
 constexpr int DD_SMEM = 4 * 3 * DD_CTA_E;       // bytes (also 16 warp regions)
-constexpr int DD_K = 4;                         // rows per thread in flight
+constexpr int DD_K = 2;                         // rows per thread per round (feature rows of 1-2 words)
 constexpr int DD_XW = NARROW_WD;                // widest feature row (words) of dedup_kernel<false>
 constexpr int DD_XW_WIDE = 16;                  // widest of dedup_kernel<true> (one row in flight)
 constexpr int DEDUP_PROBES = 8;                 // linear-probe limit
@@ -306,7 +309,7 @@ __device__ __forceinline__ void dd_sync()
 // One group of G warps finds the representatives of context c and writes
 // them, in stream order, to rep_list[row_off[c] + k] with their duplicate
 // counts in rep_dup; rep_count[c] = number of representatives.  Each thread
-// keeps DD_K rows in flight.  Table slot: (fingerprint, smallest row index
+// takes DD_K rows a round (one for feature rows of 3 or more words).  Table slot: (fingerprint, smallest row index
 // of that content) plus a duplicate counter; a full row comparison decides
 // every match, so a row is a duplicate only if it equals an earlier row.
 template <int G, int XW>
@@ -319,7 +322,6 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
     uint2* tab = reinterpret_cast<uint2*>(region);
     int* D = reinterpret_cast<int*>(region + 2 * E);
     const CtxDesc cd = s.desc[c];
-    constexpr int xw = XW;
     const int n = cd.n;
     const int64_t r0 = a.row_off[c];
     const int T = (int)(a.row_off[c + 1] - r0);
@@ -333,19 +335,9 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
     }
     dd_sync<G>();
     int nrep = 0;
-    // rows of the round in flight, and the next round's rows prefetched while
-    // the current one is probed and verified
-    constexpr int K = (XW <= 2) ? DD_K : (XW <= NARROW_WD ? 2 : 1);
-    uint4 yn[K];
-    uint32_t xn[K][XW];
-#pragma unroll
-    for (int j = 0; j < K; ++j) {
-        const int i = j * NT + t;
-        const bool ok = i < T;
-        yn[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int v = 0; v < XW; ++v) xn[j][v] = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
-    }
+    // the round's rows (no prefetch into registers: the other warps hide
+    // the load latency)
+    constexpr int K = (XW <= 2) ? DD_K : 1;
     for (int base = 0; base < T; base += NT * K) {
         int mine[K];
         uint32_t h[K];
@@ -353,17 +345,14 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
         uint32_t xv[K][XW];
 #pragma unroll
         for (int j = 0; j < K; ++j) {
-            yv[j] = yn[j];
-#pragma unroll
-            for (int v = 0; v < XW; ++v) xv[j][v] = (v == XW - 1) ? (xn[j][v] & lm) : xn[j][v];
-        }
-#pragma unroll
-        for (int j = 0; j < K; ++j) {
-            const int i = base + NT * K + j * NT + t;
+            const int i = base + j * NT + t;
             const bool ok = i < T;
-            yn[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
+            yv[j] = ok ? __ldg(yc + i) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-            for (int v = 0; v < XW; ++v) xn[j][v] = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
+            for (int v = 0; v < XW; ++v) {
+                const uint32_t w = ok ? __ldg(xc + (int64_t)i * XW + v) : 0u;
+                xv[j][v] = (v == XW - 1) ? (w & lm) : w;
+            }
         }
 #pragma unroll
         for (int j = 0; j < K; ++j) {
@@ -489,7 +478,7 @@ __device__ __forceinline__ int pow2_at_least(int v)
 
 // Pass 1 kernel: CTA-owned contexts first, then quads, then warps.
 template <bool WX>
-__global__ void __launch_bounds__(DD_THREADS, 1) dedup_kernel(StoreDev s, DedupArgs a)
+__global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(StoreDev s, DedupArgs a)
 {
     // WX: the contexts whose feature rows have DD_XW + 1 .. DD_XW_WIDE words
     constexpr int C_CTA = WX ? CLS_DDW_CTA : CLS_DD_CTA;
@@ -1637,13 +1626,13 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (e != cudaSuccess) return f2_cuda_status(e);
         cudaStream_t ks = fk.next(wide_rows ? 2 : 1);
         if (fk.e != cudaSuccess) return f2_cuda_status(fk.e);
-        dedup_kernel<false><<<st->num_sms, DD_THREADS, DD_SMEM, ks>>>(sd, da);
+        dedup_kernel<false><<<DD_CTAS_PER_SM * st->num_sms, DD_THREADS, DD_SMEM, ks>>>(sd, da);
         e = cudaGetLastError();
         if (e != cudaSuccess) return f2_cuda_status(e);
         if (wide_rows) {
             e = cudaFuncSetAttribute(dedup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
             if (e != cudaSuccess) return f2_cuda_status(e);
-            dedup_kernel<true><<<st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+            dedup_kernel<true><<<DD_CTAS_PER_SM * st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
             e = cudaGetLastError();
             if (e != cudaSuccess) return f2_cuda_status(e);
         }
