@@ -323,7 +323,7 @@ __global__ void __launch_bounds__(SCAT_THREADS) enc_scatter_kernel(int32_t Q, co
 // shared-memory region with one round of loads, then every lane reduces its
 // query against them in a warp-uniform walk over the pivots.
 // ---------------------------------------------------------------------------
-constexpr int RUN_THREADS = 256;
+constexpr int RUN_THREADS = 512;  // two CTAs per SM: 32 warps (three CTAs of 256 gave 24)
 constexpr int RUN_SEG = 2048;
 constexpr int RUN_PER = RUN_SEG / RUN_THREADS;
 constexpr int TAB_WD = NARROW_WD;             // widest context with a table (d <= 288)
@@ -363,7 +363,7 @@ struct RunSmem {
     int32_t n_groups;
     int32_t item_base;
 };
-static_assert(sizeof(RunSmem) + 1024 <= 233472 / 3, "three CTAs of enc_runs_kernel per SM");
+static_assert(sizeof(RunSmem) + 1024 <= 233472 / 2, "two CTAs of enc_runs_kernel per SM");
 
 __device__ __forceinline__ void encode_direct(const StoreDev& s, int32_t c, int64_t i, const uint32_t* __restrict__ x,
                                               int stride, uint4* __restrict__ y, uint8_t* __restrict__ in_span)
@@ -609,7 +609,7 @@ __device__ __forceinline__ void query_group(const StoreDev& s, const RunSmem& sm
     }
 }
 
-__global__ void __launch_bounds__(RUN_THREADS, 3) enc_runs_kernel(StoreDev s, int32_t n_total,
+__global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, int32_t n_total,
                                                                   const unsigned long long* __restrict__ sorted,
                                                                   const uint32_t* __restrict__ x, int stride,
                                                                   uint4* __restrict__ y,
