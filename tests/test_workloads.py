@@ -105,3 +105,22 @@ def test_parsed_lowrank_layout_and_map():
             assert flips == (1 if i == wl.contra_pos[c] else 0)
         # at most 2^(r-1) distinct x (an affine subspace of dimension r - 1)
         assert len({bytes(r) for r in xs}) <= 2 ** (int(wl.fresh[c]) - 1)
+
+
+def test_parsed_lowrank_groups_share_the_map():
+    """Consecutive contexts in groups of group_size share k and the planted
+    (A, b) (the exact contexts of one (f, m) group); different groups draw
+    their own."""
+    gs = 4
+    wl = wlmod.parsed_lowrank(num_ctx=24, seed=5, rows_per_rank=10, group_size=gs)
+    for g0 in range(0, wl.num_ctx, gs):
+        n = int(wl.n_bits[g0])
+        a0 = int(wl.a_off[g0])
+        for c in range(g0, g0 + gs):
+            assert int(wl.n_bits[c]) == n
+            ac = int(wl.a_off[c])
+            assert np.array_equal(wl.A[ac:ac + n], wl.A[a0:a0 + n])
+            assert np.array_equal(wl.b[c], wl.b[g0])
+    firsts = list(range(0, wl.num_ctx, gs))
+    maps = {(int(wl.n_bits[c]), bytes(wl.b[c])) for c in firsts}
+    assert len(maps) == len(firsts)
