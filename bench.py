@@ -559,22 +559,14 @@ def launches_per_step(wl, has_q: bool) -> int:
     call a plan (3 kernels) and dedup_kernel (a second instance when some
     feature row has more than 9 words) for the duplicate pass, a plan,
     the elimination kernel of each width class present (d <= 96, 96 < d <=
-    288, wider) and the full-rank check; solve_kernel; per 2^25 queries the
-    five encode kernels."""
+    288, 288 < d <= 544, wider) and the full-rank check; solve_kernel; per
+    2^25 queries the five encode kernels."""
     wd = (wl.n_bits.astype(np.int64) + 1 + 31) // 32
     xw = (wl.n_bits.astype(np.int64) + 31) // 32
     learn = (3 + 1 + int((xw > 9).any()) + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any())
-             + int(store_has_wide(wl)) + 1)
+             + int(((wd > 9) & (wd <= 17)).any()) + int((wd > 17).any()) + 1)
     enc = 5 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
     return len(wl.batches) * learn + 1 + enc
-
-
-def store_has_wide(wl) -> bool:
-    return bool((((wl.n_bits.astype(np.int64) + 1 + 31) // 32) > 9).any())
-
-
-def store_has_narrow(wl) -> bool:
-    return bool((((wl.n_bits.astype(np.int64) + 1 + 31) // 32) <= 9).any())
 
 
 def basis_bytes_touched(wl, store) -> int:
