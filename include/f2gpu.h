@@ -189,7 +189,10 @@ int f2_encode_batched(const f2_store* store, int64_t Q, const int32_t* ctx_id_de
  * host arrays are read asynchronously: keep them unchanged until `stream`
  * has passed the call.  Device scratch: two chunk buffers and the rebased
  * offsets (16 bytes per context), grown on demand (the call then
- * synchronizes `stream`); kept by the store until f2_destroy.
+ * synchronizes `stream`); kept by the store until f2_destroy.  Errors:
+ * F2_ERR_INVALID_ARG (NULL pointers, negative sizes, the host checks above;
+ * nothing is enqueued), F2_ERR_OOM, F2_ERR_CUDA, and those of
+ * f2_learn_batched for each chunk (device-detected ones in the status word).
  */
 int f2_learn_host(f2_store* store, const int64_t* row_off_host, const uint32_t* x_host,
                   const int64_t* x_off_host, const uint32_t* y_host, int64_t total_rows,
