@@ -166,9 +166,14 @@ int f2_solve_affine(const f2_store* store, uint32_t* W_dev, f2_stream_t stream);
  * and zero otherwise; in_span_dev[q] receives 1 (supported), 0 (rejected) or
  * 0xFF (context id out of range -- F2_ERR_CTX_RANGE is recorded -- or the
  * context needs more than x_stride_words words -- F2_ERR_STRIDE).
- * The queries are grouped by context on the device first; the store keeps
- * that scratch (20 bytes per query, at most 2^25 queries per pass, plus 4
- * bytes per context) and grows it stream-ordered with cudaMallocAsync.
+ * The queries are grouped by context on the device first, and every context
+ * with at least F2_OPT_ENCODE_TABLE_MIN queries in a pass gets a lookup table
+ * of its basis (16*ceil(d/4)*(4 + ceil((d - rank)/32)) words, for d <= 288 and
+ * d - rank <= 128).  The store keeps that scratch: 20 bytes per query (at most
+ * 2^25 queries per pass), about 8*(1 + chunks) bytes per context, and a table
+ * pool with room for the table of every context that can have one (at most
+ * 1 GiB; a context whose table does not fit is encoded without one), all
+ * allocated stream-ordered with cudaMallocAsync on first need.
  * Errors: F2_ERR_INVALID_ARG (Q < 0, NULL pointers, x_stride_words < 1),
  * F2_ERR_ALIGN (y_out_dev not 16-byte aligned), F2_ERR_OOM (scratch).
  */
@@ -282,11 +287,16 @@ enum f2_option {
     F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context */
     F2_OPT_DEDUP = 4,            /* 1 (default): eliminate only the first occurrence of each distinct
                                     row and classify its repeats with it; 0: eliminate every row */
-    F2_OPT_ENCODE_TABLE_MIN = 5, /* shortest run of queries of one context (within a block of 2,048
-                                    grouped queries) encoded with a lookup table of its basis; default
-                                    32, at least 16; a value above 2,048 disables the tables */
-    F2_OPT_HOST_CHUNK_BYTES = 6  /* bytes of rows (f2_learn_host) or of queries (f2_encode_host) per
+    F2_OPT_ENCODE_TABLE_MIN = 5, /* fewest queries of one context (in a pass of f2_encode_batched)
+                                    for which a lookup table of its basis is built; default 32, at
+                                    least 1; a value above the pass size disables the tables */
+    F2_OPT_HOST_CHUNK_BYTES = 6, /* bytes of rows (f2_learn_host) or of queries (f2_encode_host) per
                                     copied chunk; default 512 MiB, at least 64 KiB */
+    F2_OPT_ENCODE_CHUNK_SHIFT = 7, /* log2 of the consecutive queries whose table-encoded results are
+                                    written together (L2 locality of f2_encode_batched's output);
+                                    default 20, in [11, 25]; raised so a pass has at most 64 chunks */
+    F2_OPT_ENCODE_CHUNK_MIN = 8  /* fewest queries of one context (in a pass) for which its queries are
+                                    laid out chunk by chunk (the others keep one run); default 1024 */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -34,6 +34,8 @@ F2_OPT_WARP_WORK = 3
 F2_OPT_DEDUP = 4
 F2_OPT_ENCODE_TABLE_MIN = 5
 F2_OPT_HOST_CHUNK_BYTES = 6
+F2_OPT_ENCODE_CHUNK_SHIFT = 7
+F2_OPT_ENCODE_CHUNK_MIN = 8
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

@@ -3,12 +3,14 @@
 // q = phi(x) is reduced against its context's reduced basis; every stored row
 // used also XORs its z_k into a zero accumulator.  Because the basis is
 // reduced, the rows to use are exactly the pivots set in q itself.  A zero
-// residual at the non-pivot columns proves q in the span and the accumulator
+// residual at the non-pivot coordinates proves q in the span and the accumulator
 // is the word; otherwise the query is rejected and the word is zero.
 //
-// The queries are first grouped by context (pass 1 below); long runs of one
-// context are then encoded with a lookup table of its basis in shared memory
-// and the rest by a per-thread walk over the pivots set in q (pass 2).
+// The queries are first grouped by context (pass 1 below); every context
+// with many queries gets a lookup table of its basis, built once per pass in
+// a pool, and its runs of queries are encoded from that table after a bulk
+// asynchronous copy into shared memory; the other queries are encoded by a
+// per-query walk over the pivot rows staged in shared memory (pass 2).
 #include "f2_internal.cuh"
 
 using namespace f2;
@@ -95,20 +97,35 @@ __device__ __forceinline__ bool encode_one(const StoreDev& s, const CtxDesc& cd,
     return resid == 0;
 }
 
+
 // ---------------------------------------------------------------------------
-// Pass 1: group the queries by context (a counting sort; the order inside a
-// context's bucket is arbitrary, since every query's result depends only on
-// the query).  Ids outside [0, num_ctx) go to the extra bucket num_ctx.
+// Pass 1: group the queries (a counting sort; the order of the queries inside
+// a bucket is arbitrary, since every query's result depends only on the
+// query).  Ids outside [0, num_ctx) go to the extra bucket num_ctx.
 //
-//   enc_count_kernel   a CTA aggregates ENC_TILE consecutive queries per
-//                      context in a shared-memory hash table (one shared
-//                      atomic per distinct context per warp), claims each
+// A bucket is (chunk, context), a chunk being 2^shift consecutive queries.
+// The contexts that get a lookup table in this pass ("table contexts", at
+// least table_min queries) are laid out chunk-major: the encoding of a chunk
+// then reads and writes a window of the query arrays small enough to stay in
+// L2, so the words and flags scattered back to query order merge into whole
+// sectors there instead of costing a DRAM read-modify-write each.  Every
+// other context keeps its queries of all chunks together (after the table
+// contexts), so its basis is staged once.
+//
+//   enc_count_kernel   a CTA counts ENC_TILE queries (inside one chunk) per
+//                      context in a shared-memory hash table, claims each
 //                      context's share of its bucket with one global atomic,
 //                      and writes every query's offset inside its bucket;
-//   enc_scan_kernel    exclusive prefix of the bucket sizes: per tile of
-//                      SCAN_TILE buckets, then the tile totals (by the last
+//   enc_table_kernel   per context: total over the chunks; a table context
+//                      gets a slot in the store's table pool and its table
+//                      is built there (one warp); writes the scan input (the
+//                      chunk counts of table contexts, chunk-major, then the
+//                      totals of the others) and, for the others, turns the
+//                      chunk counts into their prefix over the chunks;
+//   enc_scan_kernel    exclusive prefix of the scan input: per tile of
+//                      SCAN_TILE entries, then the tile totals (by the last
 //                      CTA to finish);
-//   enc_scatter_kernel writes (bucket, query) to its bucket position.
+//   enc_scatter_kernel writes (context, query) to its grouped position.
 // ---------------------------------------------------------------------------
 constexpr int ENC_TILE = 2048;
 constexpr int ENC_TILE_THREADS = 256;
@@ -118,11 +135,20 @@ constexpr int ENC_HT = 1 << ENC_HT_BITS;
 static_assert(ENC_HT >= 2 * ENC_TILE, "hash table of a tile at most half full");
 constexpr int SCAN_THREADS = 1024;
 constexpr int SCAN_SHIFT = 12;
-constexpr int SCAN_TILE = 1 << SCAN_SHIFT;  // 4 buckets per thread
+constexpr int SCAN_TILE = 1 << SCAN_SHIFT;  // 4 entries per thread
 constexpr int SCAT_THREADS = 256;
 constexpr int SCAT_PER = 4;
 constexpr int64_t ENC_SUB = int64_t(1) << 25;   // queries grouped per pass
+constexpr int ENC_MAX_CHUNKS = 64;              // chunks of a pass (the chunk grows with the pass)
+constexpr int ENC_MIN_SHIFT = 11;               // a count tile lies inside one chunk
+constexpr int DEFAULT_CHUNK_SHIFT = 20;
 constexpr int32_t EMPTY_KEY = -1;
+constexpr int TBL_THREADS = 256;
+constexpr uint8_t HOT_TABLE = 1;    // the context's runs are encoded with its table
+constexpr uint8_t HOT_CHUNKED = 2;  // the context's queries are laid out chunk by chunk
+constexpr int64_t DEFAULT_CHUNK_MIN = 1024;
+constexpr int64_t POOL_MAX_WORDS = int64_t(1) << 28;  // table pool cap (1 GiB)
+static_assert(ENC_TILE <= (1 << ENC_MIN_SHIFT), "count tiles never straddle a chunk");
 
 __device__ __forceinline__ int32_t bucket_of(int32_t c, int32_t num_ctx)
 {
@@ -163,13 +189,15 @@ __device__ __forceinline__ T block_exclusive_scan(T v, T* ws, T& total)
 }
 
 __global__ void __launch_bounds__(ENC_TILE_THREADS) enc_count_kernel(int32_t Q, const int32_t* __restrict__ ctx_id,
-                                                                     int32_t num_ctx, int32_t* __restrict__ bins,
+                                                                     int32_t num_ctx, int shift, int32_t B,
+                                                                     int32_t* __restrict__ cnt,
                                                                      int32_t* __restrict__ off)
 {
     __shared__ int32_t key[ENC_HT];
-    __shared__ int32_t cnt[ENC_HT];
+    __shared__ int32_t hcnt[ENC_HT];
     const int t = threadIdx.x, lane = t & 31;
     const int64_t base = (int64_t)blockIdx.x * ENC_TILE;
+    int32_t* const bins = cnt + (int64_t)(base >> shift) * B;  // the tile's chunk
     int32_t bk[ENC_TILE_PER];
 #pragma unroll
     for (int j = 0; j < ENC_TILE_PER; ++j) {  // all loads first
@@ -178,31 +206,44 @@ __global__ void __launch_bounds__(ENC_TILE_THREADS) enc_count_kernel(int32_t Q, 
     }
     for (int h = t; h < ENC_HT; h += ENC_TILE_THREADS) {
         key[h] = EMPTY_KEY;
-        cnt[h] = 0;
+        hcnt[h] = 0;
     }
     __syncthreads();
     const uint32_t below = (1u << lane) - 1u;
-    int slot[ENC_TILE_PER], rank[ENC_TILE_PER];
+    uint32_t peers[ENC_TILE_PER];
+    uint32_t slot[ENC_TILE_PER];
+    int32_t prev[ENC_TILE_PER];
+    bool lead[ENC_TILE_PER];
 #pragma unroll
     for (int j = 0; j < ENC_TILE_PER; ++j) {
-        const int32_t b = bk[j];
-        const uint32_t peers = __match_any_sync(FULL, b);
-        const int leader = __ffs(peers) - 1;
-        int sl = 0, r0 = 0;
-        if (lane == leader && b != EMPTY_KEY) {
+        peers[j] = __match_any_sync(FULL, bk[j]);
+        lead[j] = lane == __ffs(peers[j]) - 1 && bk[j] != EMPTY_KEY;
+        slot[j] = ((uint32_t)bk[j] * 2654435761u) >> (32 - ENC_HT_BITS);
+    }
+    // The first probe of every group is issued before any is resolved: at
+    // most half of the table is used, so most groups are placed by it.
+#pragma unroll
+    for (int j = 0; j < ENC_TILE_PER; ++j) prev[j] = lead[j] ? atomicCAS(&key[slot[j]], EMPTY_KEY, bk[j]) : EMPTY_KEY;
+#pragma unroll
+    for (int j = 0; j < ENC_TILE_PER; ++j) {
+        if (lead[j]) {
             // at most ENC_TILE distinct keys in ENC_HT slots: a free or
             // matching slot is always found within ENC_HT probes
-            uint32_t h = ((uint32_t)b * 2654435761u) >> (32 - ENC_HT_BITS);
-            for (int probe = 0; probe < ENC_HT; ++probe) {
-                const int32_t prev = atomicCAS(&key[h], EMPTY_KEY, b);
-                if (prev == EMPTY_KEY || prev == b) break;
-                h = (h + 1) & (ENC_HT - 1);
+            for (int probe = 1; probe < ENC_HT && prev[j] != EMPTY_KEY && prev[j] != bk[j]; ++probe) {
+                slot[j] = (slot[j] + 1) & (ENC_HT - 1);
+                prev[j] = atomicCAS(&key[slot[j]], EMPTY_KEY, bk[j]);
             }
-            sl = (int)h;
-            r0 = atomicAdd(&cnt[h], __popc(peers));
         }
-        slot[j] = __shfl_sync(FULL, sl, leader);
-        rank[j] = __shfl_sync(FULL, r0, leader) + __popc(peers & below);
+    }
+    int r0[ENC_TILE_PER];
+#pragma unroll
+    for (int j = 0; j < ENC_TILE_PER; ++j) r0[j] = lead[j] ? atomicAdd(&hcnt[slot[j]], __popc(peers[j])) : 0;
+    int rank[ENC_TILE_PER];
+#pragma unroll
+    for (int j = 0; j < ENC_TILE_PER; ++j) {
+        const int leader = __ffs(peers[j]) - 1;
+        slot[j] = __shfl_sync(FULL, slot[j], leader);
+        rank[j] = __shfl_sync(FULL, r0[j], leader) + __popc(peers[j] & below);
     }
     __syncthreads();
     // one global atomic per distinct context of the tile; all of a thread's
@@ -213,16 +254,266 @@ __global__ void __launch_bounds__(ENC_TILE_THREADS) enc_count_kernel(int32_t Q, 
     for (int u = 0; u < HPER; ++u) {
         const int h = u * ENC_TILE_THREADS + t;
         const int32_t k = key[h];
-        got[u] = (k != EMPTY_KEY) ? atomicAdd(bins + k, cnt[h]) : 0;
+        got[u] = (k != EMPTY_KEY) ? atomicAdd(bins + k, hcnt[h]) : 0;
     }
     __syncthreads();
 #pragma unroll
-    for (int u = 0; u < HPER; ++u) cnt[u * ENC_TILE_THREADS + t] = got[u];
+    for (int u = 0; u < HPER; ++u) hcnt[u * ENC_TILE_THREADS + t] = got[u];
     __syncthreads();
 #pragma unroll
     for (int j = 0; j < ENC_TILE_PER; ++j) {
         const int64_t i = base + (int64_t)j * ENC_TILE_THREADS + t;
-        if (i < Q) off[i] = cnt[slot[j]] + rank[j];
+        if (i < Q) off[i] = hcnt[slot[j]] + rank[j];
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Lookup tables (a Four-Russians table over 4-bit groups of coordinates).
+// The reduction of q against the reduced basis XORs, for every set
+// coordinate j of q, the vector E_j:
+//   j a pivot:     word part z_j, residual part r_j restricted to the
+//                  non-pivot coordinates (r_j has no other pivot bit);
+//   j not a pivot: word part 0, residual part the unit vector of j.
+// Residuals live on the m = d - rank non-pivot coordinates only, so they are
+// stored compressed (the t-th non-pivot coordinate in increasing order is
+// bit t).  E is linear in q, so for each group p of four coordinates the
+// table holds all 16 XOR combinations of E_{4p..4p+3}; a query then costs
+// exactly ceil(d/4) lookups and is in the span iff its compressed residual is
+// zero (Sec. 2.3: the word is T(q) = XOR of the z_k used; the query is
+// rejected otherwise).
+//
+// Layout of a table with np groups and rw residual words (word offsets):
+// low z half uint2[np*16] at 0, high z half at 32*np, residual word u
+// uint32[np*16] at 64*np + 16*np*u; entry e = 16*p + v.  With eight-byte and
+// four-byte planes the lookups of a warp at one position are free of bank
+// conflicts (the 16 values of v fall in distinct banks).  A table is
+// 16*np*(4 + rw) words, a multiple of 64 bytes.
+// ---------------------------------------------------------------------------
+constexpr int TAB_WD = NARROW_WD;             // widest context with a table (d <= 288)
+constexpr int TAB_RW = 4;                     // compressed residual words (m <= 128)
+constexpr int TAB_WORDS = 6144;               // largest table (24 KB): one of two table buffers
+constexpr int DEFAULT_TABLE_MIN = 32;
+
+__host__ __device__ __forceinline__ int table_words(int d, int rank)
+{
+    const int np = (d + 3) >> 2, rw = (d - rank + 31) >> 5;
+    return 16 * np * (4 + rw);
+}
+
+// E_j of context cd: word part z, compressed residual er.  The pivot words,
+// z_j and r_j are loaded together (slots of non-pivots hold zeros), so an
+// entry costs one round of loads.
+__device__ __forceinline__ void single_entry(const StoreDev& s, const CtxDesc& cd, int j, uint4& z,
+                                             uint32_t (&er)[TAB_RW])
+{
+#pragma unroll
+    for (int u = 0; u < TAB_RW; ++u) er[u] = 0;
+    z = make_uint4(0, 0, 0, 0);
+    if (j >= cd.d) return;
+    const uint32_t* __restrict__ P = s.pivot + cd.pw_off;
+    const uint32_t* __restrict__ row = s.bx + cd.xw_off + (int64_t)j * cd.wd;
+    const int w = j >> 5, b = j & 31;
+    uint32_t pv[TAB_WD], rv[TAB_WD];
+#pragma unroll
+    for (int u = 0; u < TAB_WD; ++u) {
+        pv[u] = (u <= w) ? __ldg(P + u) : 0u;
+        rv[u] = (u <= w) ? __ldg(row + u) : 0u;
+    }
+    const uint4 zj = __ldg(s.bz + cd.slot_off + j);
+    auto set_bit = [&](int t) {
+#pragma unroll
+        for (int u = 0; u < TAB_RW; ++u)
+            if ((t >> 5) == u) er[u] |= 1u << (t & 31);
+    };
+    int below = 0;  // non-pivot coordinates in the words before u (all full: u < w <= wd - 1)
+    bool pivot = false;
+#pragma unroll
+    for (int u = 0; u < TAB_WD; ++u) {
+        if (u == w) pivot = (pv[u] >> b) & 1u;
+    }
+    if (pivot) {
+        z = zj;
+#pragma unroll
+        for (int u = 0; u < TAB_WD; ++u) {
+            if (u <= w) {
+                const uint32_t free_u = ~pv[u];
+                uint32_t bits = rv[u] & free_u;  // r_j has no bit above j
+                while (bits) {
+                    const int bb = __ffs(bits) - 1;
+                    set_bit(below + __popc(free_u & ((1u << bb) - 1u)));
+                    bits &= bits - 1u;
+                }
+                below += __popc(free_u);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int u = 0; u < TAB_WD; ++u) {
+            if (u < w) below += __popc(~pv[u]);
+            if (u == w) set_bit(below + __popc(~pv[u] & ((1u << b) - 1u)));
+        }
+    }
+}
+
+// One warp writes block blk (coordinates 32*blk .. 32*blk + 31, i.e. eight
+// groups) of the table of context c to `tab` (global memory).  Lane l
+// computes E_j for j = 32*blk + l; the four lanes of a quad hold the four
+// coordinates of one group and each writes four of its 16 entries (entry v
+// = XOR of E_{4p+b} over the bits b of v).
+__device__ void build_table(const StoreDev& s, int c, int blk, uint32_t* __restrict__ tab, int lane)
+{
+    const CtxDesc cd = s.desc[c];
+    const int rank = s.rank[c];
+    const int np = (cd.d + 3) >> 2, rw = (cd.d - rank + 31) >> 5;
+    uint2* const Zl = reinterpret_cast<uint2*>(tab);
+    uint2* const Zh = Zl + 16 * np;
+    uint32_t* const R = tab + 64 * np;
+    const int qb = lane & ~3, b = lane & 3;
+    {
+        const int j = 32 * blk + lane;
+        uint4 z;
+        uint32_t er[TAB_RW];
+        single_entry(s, cd, j, z, er);
+        uint4 zs[4];
+        uint32_t es[4][TAB_RW];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            zs[k].x = __shfl_sync(FULL, z.x, qb + k);
+            zs[k].y = __shfl_sync(FULL, z.y, qb + k);
+            zs[k].z = __shfl_sync(FULL, z.z, qb + k);
+            zs[k].w = __shfl_sync(FULL, z.w, qb + k);
+#pragma unroll
+            for (int u = 0; u < TAB_RW; ++u) es[k][u] = __shfl_sync(FULL, er[u], qb + k);
+        }
+        if (j < 4 * np) {
+            // entries v = 4b .. 4b+3 of group p: 32 contiguous bytes per z
+            // plane and 16 per residual plane, written as whole 16-byte stores
+            const int p = j >> 2;
+            uint4 a[4];
+            uint32_t ra[4][TAB_RW];
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                const int v = 4 * b + m;
+                a[m] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int u = 0; u < TAB_RW; ++u) ra[m][u] = 0;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    if ((v >> k) & 1) {
+                        a[m].x ^= zs[k].x;
+                        a[m].y ^= zs[k].y;
+                        a[m].z ^= zs[k].z;
+                        a[m].w ^= zs[k].w;
+#pragma unroll
+                        for (int u = 0; u < TAB_RW; ++u) ra[m][u] ^= es[k][u];
+                    }
+                }
+            }
+            const int e = 16 * p + 4 * b;
+            uint4* zl = reinterpret_cast<uint4*>(Zl + e);
+            uint4* zh = reinterpret_cast<uint4*>(Zh + e);
+            zl[0] = make_uint4(a[0].x, a[0].y, a[1].x, a[1].y);
+            zl[1] = make_uint4(a[2].x, a[2].y, a[3].x, a[3].y);
+            zh[0] = make_uint4(a[0].z, a[0].w, a[1].z, a[1].w);
+            zh[1] = make_uint4(a[2].z, a[2].w, a[3].z, a[3].w);
+#pragma unroll
+            for (int u = 0; u < TAB_RW; ++u)
+                if (u < rw)
+                    *reinterpret_cast<uint4*>(R + u * 16 * np + e) = make_uint4(ra[0][u], ra[1][u], ra[2][u], ra[3][u]);
+        }
+    }
+}
+
+// Per bucket b (a thread; consecutive buckets, so the chunk counts are read
+// coalesced): its total over the chunks; table or not (a slot in the pool,
+// claimed once per warp); the scan input; the table contexts are listed for
+// enc_build_kernel.
+__global__ void __launch_bounds__(TBL_THREADS) enc_table_kernel(StoreDev s, int32_t nch, int32_t B,
+                                                                int32_t* __restrict__ cnt,
+                                                                int32_t* __restrict__ scan_in,
+                                                                uint8_t* __restrict__ hot,
+                                                                long long* __restrict__ tab_off,
+                                                                long long pool_words,
+                                                                unsigned long long* __restrict__ pool_used,
+                                                                int32_t* __restrict__ hot_list,
+                                                                int32_t* __restrict__ n_hot, int table_min,
+                                                                long long chunk_min, int stride)
+{
+    const int lane = threadIdx.x & 31;
+    for (int c0 = (int)((blockIdx.x * (unsigned)TBL_THREADS + threadIdx.x) & ~31u); c0 < B;
+         c0 += (int)(gridDim.x * (unsigned)TBL_THREADS)) {
+        const int c = c0 + lane;
+        int tot = 0, words = 0;
+        if (c < B)
+            for (int ch = 0; ch < nch; ++ch) tot += cnt[(int64_t)ch * B + c];
+        if (c < s.num_ctx && tot >= table_min) {
+            const CtxDesc cd = s.desc[c];
+            const int rk = s.rank[c];
+            const int w = table_words(cd.d, rk);
+            const int rw = (cd.d - rk + 31) >> 5;
+            if (cd.wd <= TAB_WD && cd.xw <= stride && rw <= TAB_RW && w <= TAB_WORDS) words = w;
+        }
+        // one pool claim and one list claim per warp
+        int incl = words;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(FULL, incl, o);
+            if (lane >= o) incl += u;
+        }
+        const int wsum = __shfl_sync(FULL, incl, 31);
+        unsigned long long wbase = 0;
+        if (lane == 31 && wsum) wbase = atomicAdd(pool_used, (unsigned long long)wsum);
+        wbase = __shfl_sync(FULL, wbase, 31);
+        const long long o = (long long)wbase + incl - words;
+        const bool h = words > 0 && o + words <= pool_words;
+        // the table's blocks of 32 coordinates are listed for enc_build_kernel
+        const int nb = h ? (((s.desc[c].d + 3) >> 2) * 4 + 31) >> 5 : 0;
+        int binc = nb;
+#pragma unroll
+        for (int o2 = 1; o2 < 32; o2 <<= 1) {
+            const int u = __shfl_up_sync(FULL, binc, o2);
+            if (lane >= o2) binc += u;
+        }
+        const int bsum = __shfl_sync(FULL, binc, 31);
+        int lbase = 0;
+        if (lane == 31 && bsum) lbase = atomicAdd(n_hot, bsum);
+        lbase = __shfl_sync(FULL, lbase, 31);
+        for (int k = 0; k < nb; ++k) hot_list[lbase + binc - nb + k] = (int32_t)(((uint32_t)c << 4) | (uint32_t)k);
+        if (c < B) {
+            const bool chunked = c < s.num_ctx && (long long)tot >= chunk_min;
+            hot[c] = (h ? HOT_TABLE : 0) | (chunked ? HOT_CHUNKED : 0);
+            tab_off[c] = h ? o : -1;
+            if (chunked) {
+                for (int ch = 0; ch < nch; ++ch) scan_in[(int64_t)ch * B + c] = cnt[(int64_t)ch * B + c];
+                scan_in[(int64_t)nch * B + c] = 0;
+            } else {
+                int run = 0;
+                for (int ch = 0; ch < nch; ++ch) {
+                    const int v = cnt[(int64_t)ch * B + c];
+                    scan_in[(int64_t)ch * B + c] = 0;
+                    cnt[(int64_t)ch * B + c] = run;  // the bucket's queries before chunk ch
+                    run += v;
+                }
+                scan_in[(int64_t)nch * B + c] = tot;
+            }
+        }
+    }
+}
+
+// A warp per listed (table context, block of 32 coordinates) builds that
+// part of the context's table in the pool.
+__global__ void __launch_bounds__(TBL_THREADS) enc_build_kernel(StoreDev s, const int32_t* __restrict__ hot_list,
+                                                                const int32_t* __restrict__ n_hot,
+                                                                const long long* __restrict__ tab_off,
+                                                                uint32_t* __restrict__ pool)
+{
+    const int lane = threadIdx.x & 31;
+    const int nh = *n_hot;
+    const int nw = (int)((gridDim.x * (unsigned)TBL_THREADS) >> 5);
+    for (int k = (int)((blockIdx.x * (unsigned)TBL_THREADS + threadIdx.x) >> 5); k < nh; k += nw) {
+        const uint32_t item = (uint32_t)__ldg(hot_list + k);
+        const int c = (int)(item >> 4);
+        build_table(s, c, (int)(item & 15u), pool + __ldg(tab_off + c), lane);
     }
 }
 
@@ -271,9 +562,18 @@ __global__ void __launch_bounds__(SCAN_THREADS) enc_scan_kernel(int32_t* __restr
     }
 }
 
+__device__ __forceinline__ int32_t scan_start(const int32_t* __restrict__ sta, const int32_t* __restrict__ tpre,
+                                              int64_t k)
+{
+    return __ldg(sta + k) + __ldg(tpre + (k >> SCAN_SHIFT));
+}
+
 __global__ void __launch_bounds__(SCAT_THREADS) enc_scatter_kernel(int32_t Q, const int32_t* __restrict__ ctx_id,
-                                                                   int32_t num_ctx, const int32_t* __restrict__ bins,
+                                                                   int32_t num_ctx, int shift, int32_t nch, int32_t B,
+                                                                   const int32_t* __restrict__ cnt,
+                                                                   const int32_t* __restrict__ sta,
                                                                    const int32_t* __restrict__ tpre,
+                                                                   const uint8_t* __restrict__ hot,
                                                                    const int32_t* __restrict__ off,
                                                                    unsigned long long* __restrict__ sorted)
 {
@@ -288,8 +588,13 @@ __global__ void __launch_bounds__(SCAT_THREADS) enc_scatter_kernel(int32_t Q, co
     int32_t p[SCAT_PER];
 #pragma unroll
     for (int j = 0; j < SCAT_PER; ++j) {
+        const int64_t i = base + (int64_t)j * SCAT_THREADS;
         const int bb = b[j] < 0 ? 0 : b[j];
-        p[j] = __ldg(bins + bb) + __ldg(tpre + (bb >> SCAN_SHIFT)) + o[j];
+        const int64_t ch = i >> shift;
+        if (__ldg(hot + bb) & HOT_CHUNKED)
+            p[j] = scan_start(sta, tpre, ch * B + bb) + o[j];
+        else
+            p[j] = scan_start(sta, tpre, (int64_t)nch * B + bb) + __ldg(cnt + ch * B + bb) + o[j];
     }
 #pragma unroll
     for (int j = 0; j < SCAT_PER; ++j) {
@@ -303,67 +608,54 @@ __global__ void __launch_bounds__(SCAT_THREADS) enc_scatter_kernel(int32_t Q, co
 //
 // enc_runs_kernel: a CTA takes RUN_SEG consecutive positions of the grouped
 // order, i.e. a few runs of queries of one context each.  A run of at least
-// table_min queries whose context fits the tables is encoded with a table of
-// its basis (a Four-Russians table over 4-bit groups of coordinates).  The
-// reduction of q against the reduced basis XORs, for every set coordinate j
-// of q, the vector E_j:
-//   j a pivot:     word part z_j, residual part r_j restricted to the
-//                  non-pivot coordinates (r_j has no other pivot bit);
-//   j not a pivot: word part 0, residual part the unit vector of j.
-// Residuals live on the m = d - rank non-pivot coordinates only, so they are
-// stored compressed (the t-th non-pivot coordinate in increasing order is
-// bit t).  E is linear in q, so for each group p of four coordinates the
-// table holds all 16 XOR combinations of E_{4p..4p+3}; a query then costs
-// exactly ceil(d/4) lookups and is in the span iff its compressed residual is
-// zero (Sec. 2.3: the word is T(q) = XOR of the z_k used; the query is
-// rejected otherwise).  The other runs are cut into items of at most 32
-// queries and appended to a list for enc_short_kernel.
+// RUN_TABLE_MIN queries of a table context is encoded with its table: the
+// CTA copies the tables of its runs from the pool into shared memory with
+// bulk asynchronous copies (two buffers: the next group of tables is in
+// flight while the queries of the current group are looked up).  The other
+// runs are cut into items of at most 32 queries for enc_short_kernel.
 //
-// enc_short_kernel: a warp per item stages the context's basis rows in its
-// shared-memory region with one round of loads, then every lane reduces its
+// enc_short_kernel: a warp per item stages the context's pivot rows in its
+// shared-memory region with asynchronous copies, then every lane reduces its
 // query against them in a warp-uniform walk over the pivots.
 // ---------------------------------------------------------------------------
-constexpr int RUN_THREADS = 512;  // two CTAs per SM: 32 warps (three CTAs of 256 gave 24)
+constexpr int RUN_THREADS = 512;  // two CTAs per SM: 32 warps
 constexpr int RUN_SEG = 2048;
 constexpr int RUN_PER = RUN_SEG / RUN_THREADS;
-constexpr int TAB_WD = NARROW_WD;             // widest context with a table (d <= 288)
-constexpr int TAB_RW = 4;                     // compressed residual words (m <= 128)
-constexpr int TAB_WORDS = 8192;               // one group of tables (32 KB); larger tables are not built
-constexpr int MAX_TRUNS = 128;                // table runs of a segment: table_min >= RUN_SEG / MAX_TRUNS
-constexpr int DEFAULT_TABLE_MIN = 32;
+constexpr int MAX_TRUNS = 128;                // table runs of a segment (the rest become items)
+constexpr int RUN_TABLE_MIN = 4;              // shorter runs of a table context become items
+constexpr int XS_WORDS = 4;                   // feature words of a table query staged in shared memory
 constexpr int ITEM_MAX = 32;                  // queries of a short item (one per lane)
 constexpr int ITEM_POS_BITS = 25;             // item = position | (length - 1) << 25
 static_assert(ENC_SUB <= (int64_t(1) << ITEM_POS_BITS), "item positions fit 25 bits");
 
 struct RunSmem {
-    uint4 table[TAB_WORDS / 4];
-    unsigned long long ent[RUN_SEG];   // (bucket << 32) | query index
+    uint4 table[2][TAB_WORDS / 4];     // two table buffers
+    uint4 xs[RUN_SEG];                 // first XS_WORDS feature words of each table query (flat order);
+                                       // until they are staged, its first RUN_SEG words hold each run's context
+    uint32_t idx[RUN_SEG];             // query index of each position
     uint32_t flat[RUN_SEG];            // table positions in order: position | table run << 16
     uint16_t starts[RUN_SEG + 1];      // run starts
     int16_t run_tr[RUN_SEG];           // table run of each run, -1 if none
-    int32_t tr_ctx[MAX_TRUNS];
-    int32_t tr_tab[MAX_TRUNS];         // word offset of the run's table in `table`
-    int32_t tr_j0[MAX_TRUNS];          // first single-coordinate item of the run in its group
-    int32_t tr_e0[MAX_TRUNS];          // first table entry of the run in its group
+    long long tr_src[MAX_TRUNS];       // word offset of the run's table in the pool
+    int32_t tr_tab[MAX_TRUNS];         // word offset of the run's table in its buffer
+    int32_t tr_words[MAX_TRUNS];
     int32_t tr_flat[MAX_TRUNS + 1];    // first flat index of the run
-    long long tr_slot_off[MAX_TRUNS];  // the run's context: basis offsets
-    long long tr_xw_off[MAX_TRUNS];
-    long long tr_pw_off[MAX_TRUNS];
-    int16_t tr_d[MAX_TRUNS];
-    uint8_t tr_wd[MAX_TRUNS];
     int16_t tr_n[MAX_TRUNS];           // feature bits of the run's context
     uint8_t tr_np[MAX_TRUNS];
     uint8_t tr_rw[MAX_TRUNS];
     uint8_t tr_xw[MAX_TRUNS];
     int32_t g_first[MAX_TRUNS + 1];
-    int32_t g_j[MAX_TRUNS];
-    int32_t g_e[MAX_TRUNS];
     uint8_t g_xw[MAX_TRUNS];           // widest feature vector of the group's runs
+    unsigned long long bar[2];         // completion of the copies into table[0] / table[1]
     int32_t ws[RUN_THREADS / 32 + 1];
     int32_t n_groups;
     int32_t item_base;
+    int32_t failed;
 };
 static_assert(sizeof(RunSmem) + 1024 <= 233472 / 2, "two CTAs of enc_runs_kernel per SM");
+static_assert(offsetof(RunSmem, table) % 16 == 0 && offsetof(RunSmem, xs) % 16 == 0 &&
+                  offsetof(RunSmem, bar) % 8 == 0,
+              "aligned buffers");
 
 __device__ __forceinline__ void encode_direct(const StoreDev& s, int32_t c, int64_t i, const uint32_t* __restrict__ x,
                                               int stride, uint4* __restrict__ y, uint8_t* __restrict__ in_span)
@@ -424,7 +716,7 @@ __device__ __forceinline__ void load_x(const uint32_t* __restrict__ xq, int xw, 
 #pragma unroll
         for (int v4 = 0; v4 * 4 < XW; ++v4) {
             uint4 p = make_uint4(0, 0, 0, 0);
-            if (4 * v4 < xw) p = __ldg(reinterpret_cast<const uint4*>(xq) + v4);
+            if (4 * v4 < xw) p = __ldcs(reinterpret_cast<const uint4*>(xq) + v4);
             const uint32_t w[4] = {p.x, p.y, p.z, p.w};
 #pragma unroll
             for (int u = 0; u < 4; ++u)
@@ -432,70 +724,10 @@ __device__ __forceinline__ void load_x(const uint32_t* __restrict__ xq, int xw, 
         }
     } else {
 #pragma unroll
-        for (int v = 0; v < XW; ++v) xo[v] = (v < xw) ? __ldg(xq + v) : 0u;
+        for (int v = 0; v < XW; ++v) xo[v] = (v < xw) ? __ldcs(xq + v) : 0u;
     }
 }
 
-// E_j (see above) of context cd: word part z, compressed residual er.  The
-// pivot words, z_j and r_j are loaded together (slots of non-pivots hold
-// zeros), so a table costs one round of loads.
-__device__ __forceinline__ void single_entry(const StoreDev& s, const CtxDesc& cd, int j, uint4& z,
-                                             uint32_t (&er)[TAB_RW])
-{
-#pragma unroll
-    for (int u = 0; u < TAB_RW; ++u) er[u] = 0;
-    z = make_uint4(0, 0, 0, 0);
-    if (j >= cd.d) return;
-    const uint32_t* __restrict__ P = s.pivot + cd.pw_off;
-    const uint32_t* __restrict__ row = s.bx + cd.xw_off + (int64_t)j * cd.wd;
-    const int w = j >> 5, b = j & 31;
-    uint32_t pv[TAB_WD], rv[TAB_WD];
-#pragma unroll
-    for (int u = 0; u < TAB_WD; ++u) {
-        pv[u] = (u <= w) ? __ldg(P + u) : 0u;
-        rv[u] = (u <= w) ? __ldg(row + u) : 0u;
-    }
-    const uint4 zj = __ldg(s.bz + cd.slot_off + j);
-    auto set_bit = [&](int t) {
-#pragma unroll
-        for (int u = 0; u < TAB_RW; ++u)
-            if ((t >> 5) == u) er[u] |= 1u << (t & 31);
-    };
-    int below = 0;  // non-pivot coordinates in the words before u (all full: u < w <= wd - 1)
-    bool pivot = false;
-#pragma unroll
-    for (int u = 0; u < TAB_WD; ++u) {
-        if (u == w) pivot = (pv[u] >> b) & 1u;
-    }
-    if (pivot) {
-        z = zj;
-#pragma unroll
-        for (int u = 0; u < TAB_WD; ++u) {
-            if (u <= w) {
-                const uint32_t free_u = ~pv[u];
-                uint32_t bits = rv[u] & free_u;  // r_j has no bit above j
-                while (bits) {
-                    const int bb = __ffs(bits) - 1;
-                    set_bit(below + __popc(free_u & ((1u << bb) - 1u)));
-                    bits &= bits - 1u;
-                }
-                below += __popc(free_u);
-            }
-        }
-    } else {
-#pragma unroll
-        for (int u = 0; u < TAB_WD; ++u) {
-            if (u < w) below += __popc(~pv[u]);
-            if (u == w) set_bit(below + __popc(~pv[u] & ((1u << b) - 1u)));
-        }
-    }
-}
-
-// Table layout of one run with np groups and rw residual words (word
-// offsets): low z half uint2[np*16] at 0, high z half at 32*np, residual word
-// u uint32[np*16] at 64*np + 16*np*u; entry e = 16*p + v.  With eight-byte
-// and four-byte planes the lookups of a warp at one position are free of bank
-// conflicts (the 16 values of v fall in distinct banks).
 template <int RW, int WD>
 __device__ __forceinline__ bool table_query(const uint32_t* tab, int np, uint32_t (&q)[WD], uint4& acc)
 {
@@ -538,59 +770,26 @@ __device__ __forceinline__ bool table_query(const uint32_t* tab, int np, uint32_
     return res == 0;
 }
 
-// largest i in [lo, hi] with a[i] <= f (a[lo] <= f)
-__device__ __forceinline__ int find_item(const int32_t* a, int lo, int hi, int f)
-{
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (a[mid] <= f)
-            lo = mid;
-        else
-            hi = mid - 1;
-    }
-    return lo;
-}
-
 // Encode the queries at flat positions [fa, fb) of a segment with their
-// runs' tables.  A query's feature words (at most XW) are fetched PF queries
-// ahead of its lookups, so PF loads of each thread are in flight.
-template <int WD, int XW, int PF>
+// runs' tables; the first XS_WORDS feature words of each are in sm.xs.
+template <int WD>
 __device__ __forceinline__ void query_group(const StoreDev& s, const RunSmem& sm, const uint32_t* table,
-                                            const uint32_t* __restrict__ x, int stride, bool xvec,
-                                            uint4* __restrict__ y, uint8_t* __restrict__ in_span, int fa, int fb)
+                                            const uint32_t* __restrict__ x, int stride, uint4* __restrict__ y,
+                                            uint8_t* __restrict__ in_span, int fa, int fb)
 {
-    const int t = threadIdx.x;
-    uint32_t xr[PF][XW];
-    int64_t iq[PF];
-    int trq[PF];
-    auto fetch = [&](int kk, uint32_t (&xo)[XW], int64_t& i, int& tr) {
-        tr = 0;
-        i = 0;
-        int xw = 0;
-        if (kk < fb) {
-            const uint32_t fv = sm.flat[kk];
-            tr = (int)(fv >> 16);
-            i = (int64_t)(uint32_t)sm.ent[fv & 0xFFFFu];
-            xw = sm.tr_xw[tr];
-        }
-        load_x<XW>(x + i * stride, xw, xvec, xo);
-    };
-#pragma unroll
-    for (int p = 0; p < PF; ++p) fetch(fa + t + p * RUN_THREADS, xr[p], iq[p], trq[p]);
-    for (int k = fa + t; k < fb; k += RUN_THREADS) {
+    for (int f = fa + (int)threadIdx.x; f < fb; f += RUN_THREADS) {
+        const uint32_t fv = sm.flat[f];
+        const int tr = (int)(fv >> 16);
+        const int64_t i = (int64_t)sm.idx[fv & 0xFFFFu];
+        const int xw = sm.tr_xw[tr];
+        const uint4 p = sm.xs[f];
+        const uint32_t w4[4] = {p.x, p.y, p.z, p.w};
         uint32_t raw[WD];
 #pragma unroll
-        for (int v = 0; v < WD; ++v) raw[v] = (v < XW) ? xr[0][v] : 0u;
-        const int tr = trq[0];
-        const int64_t i = iq[0];
-#pragma unroll
-        for (int p = 0; p + 1 < PF; ++p) {
-#pragma unroll
-            for (int v = 0; v < XW; ++v) xr[p][v] = xr[p + 1][v];
-            iq[p] = iq[p + 1];
-            trq[p] = trq[p + 1];
+        for (int v = 0; v < WD; ++v) {
+            if (v < XS_WORDS) raw[v] = (v < xw) ? w4[v] : 0u;
+            else raw[v] = (v < xw) ? __ldcs(x + i * stride + v) : 0u;
         }
-        fetch(k + PF * RUN_THREADS, xr[PF - 1], iq[PF - 1], trq[PF - 1]);
         uint32_t q[WD];
         make_q<WD>(s.raw != 0, sm.tr_n[tr], raw, q);
         const uint32_t* tab = table + sm.tr_tab[tr];
@@ -613,37 +812,52 @@ __global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, in
                                                                   const unsigned long long* __restrict__ sorted,
                                                                   const uint32_t* __restrict__ x, int stride,
                                                                   uint4* __restrict__ y,
-                                                                  uint8_t* __restrict__ in_span, int table_min,
+                                                                  uint8_t* __restrict__ in_span,
+                                                                  const uint8_t* __restrict__ hot,
+                                                                  const long long* __restrict__ tab_off,
+                                                                  const uint32_t* __restrict__ pool,
                                                                   unsigned long long* __restrict__ items,
                                                                   int32_t* __restrict__ n_items)
 {
     extern __shared__ uint4 enc_smem[];
     RunSmem& sm = *reinterpret_cast<RunSmem*>(enc_smem);
-    uint32_t* const table = reinterpret_cast<uint32_t*>(sm.table);
+    int32_t* const run_ctx = reinterpret_cast<int32_t*>(sm.xs);  // until the feature words are staged
     const int t = threadIdx.x;
     const bool xvec = ((uintptr_t)x % 16) == 0 && (stride % 4) == 0;
     const int64_t seg0 = (int64_t)blockIdx.x * RUN_SEG;
     const int n = (int)((n_total - seg0) < RUN_SEG ? (n_total - seg0) : RUN_SEG);
-    for (int k = t; k < n; k += RUN_THREADS) sm.ent[k] = __ldg(sorted + seg0 + k);
-    __syncthreads();
-
-    // runs: flag the first position of each run, number the runs
+    if (t == 0) {
+        mbar_init(&sm.bar[0], 1);
+        mbar_init(&sm.bar[1], 1);
+        mbar_init_fence();
+        sm.failed = 0;
+    }
+    // this thread's positions: contexts in registers, query indices to smem
     const int k0 = t * RUN_PER;
+    uint32_t cx[RUN_PER];
+    uint32_t prev = 0xFFFFFFFFu;
+    if (k0 > 0 && k0 <= n) prev = (uint32_t)(__ldcs(sorted + seg0 + k0 - 1) >> 32);
+#pragma unroll
+    for (int m = 0; m < RUN_PER; ++m) {
+        const int k = k0 + m;
+        cx[m] = 0xFFFFFFFFu;
+        if (k < n) {
+            const unsigned long long e = __ldcs(sorted + seg0 + k);
+            cx[m] = (uint32_t)(e >> 32);
+            sm.idx[k] = (uint32_t)e;
+        }
+    }
+    // runs: flag the first position of each run, number the runs
     uint32_t first = 0;
     int nflag = 0;
-    {
-        uint32_t prev = (k0 > 0 && k0 <= n) ? (uint32_t)(sm.ent[k0 - 1] >> 32) : 0xFFFFFFFFu;
 #pragma unroll
-        for (int m = 0; m < RUN_PER; ++m) {
-            const int k = k0 + m;
-            if (k < n) {
-                const uint32_t b = (uint32_t)(sm.ent[k] >> 32);
-                if (k == 0 || b != prev) {
-                    first |= 1u << m;
-                    ++nflag;
-                }
-                prev = b;
+    for (int m = 0; m < RUN_PER; ++m) {
+        if (k0 + m < n) {
+            if (k0 + m == 0 || cx[m] != prev) {
+                first |= 1u << m;
+                ++nflag;
             }
+            prev = cx[m];
         }
     }
     int n_runs;
@@ -652,55 +866,52 @@ __global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, in
         int r = r0;
 #pragma unroll
         for (int m = 0; m < RUN_PER; ++m)
-            if ((first >> m) & 1u) sm.starts[r++] = (uint16_t)(k0 + m);
+            if ((first >> m) & 1u) {
+                sm.starts[r] = (uint16_t)(k0 + m);
+                run_ctx[r++] = (int32_t)cx[m];
+            }
         if (t == 0) sm.starts[n_runs] = (uint16_t)n;
     }
     __syncthreads();
 
     // classify the runs, RUN_THREADS at a time: number the table runs (in
-    // position order), count the items of the others
+    // position order; those past MAX_TRUNS become items), count the items
     int n_tr = 0, n_it = 0, my_base = 0;
     for (int c0 = 0; c0 < n_runs; c0 += RUN_THREADS) {
         const int rr = c0 + t;
-        int nel = 0, nit = 0, len = 0;
+        int nel = 0, len = 0;
         int32_t c = s.num_ctx;
-        CtxDesc cd{};
-        int32_t rk = 0;
         if (rr < n_runs) {
             len = (int)sm.starts[rr + 1] - (int)sm.starts[rr];
-            c = (int32_t)(sm.ent[sm.starts[rr]] >> 32);
-            if (c < s.num_ctx) {
-                cd = s.desc[c];
-                rk = s.rank[c];
-            }
-            const int np = (cd.d + 3) >> 2, rw = (cd.d - rk + 31) >> 5;
-            const bool ok = len >= table_min && c < s.num_ctx && cd.wd <= TAB_WD && cd.xw <= stride &&
-                            rw <= TAB_RW && 16 * np * (4 + rw) <= TAB_WORDS;
-            nel = ok ? 1 : 0;
-            nit = ok ? 0 : (len + ITEM_MAX - 1) / ITEM_MAX;
+            c = run_ctx[rr];
+            nel = (c < s.num_ctx && len >= RUN_TABLE_MIN && (__ldg(hot + c) & HOT_TABLE)) ? 1 : 0;
         }
         int tot;
-        const int ex = block_exclusive_scan<RUN_THREADS>(nel | (nit << 16), sm.ws, tot);
+        const int ex = block_exclusive_scan<RUN_THREADS>(nel, sm.ws, tot);
         if (rr < n_runs) {
-            if (nel) {
-                const int tr = n_tr + (ex & 0xFFFF);
+            const int tr = n_tr + ex;
+            if (nel && tr < MAX_TRUNS) {
+                const CtxDesc cd = s.desc[c];
+                const int rk = s.rank[c];
                 sm.run_tr[rr] = (int16_t)tr;
-                sm.tr_ctx[tr] = c;
                 sm.tr_np[tr] = (uint8_t)((cd.d + 3) >> 2);
                 sm.tr_rw[tr] = (uint8_t)((cd.d - rk + 31) >> 5);
                 sm.tr_xw[tr] = (uint8_t)cd.xw;
                 sm.tr_n[tr] = (int16_t)cd.n;
-                sm.tr_d[tr] = (int16_t)cd.d;
-                sm.tr_wd[tr] = (uint8_t)cd.wd;
-                sm.tr_slot_off[tr] = cd.slot_off;
-                sm.tr_xw_off[tr] = cd.xw_off;
-                sm.tr_pw_off[tr] = cd.pw_off;
+                sm.tr_words[tr] = table_words(cd.d, rk);
+                sm.tr_src[tr] = __ldg(tab_off + c);
             } else {
                 sm.run_tr[rr] = -1;
+                n_it += (len + ITEM_MAX - 1) / ITEM_MAX;  // this thread's items
             }
         }
-        n_tr += tot & 0xFFFF;
-        n_it += tot >> 16;
+        n_tr += tot;
+    }
+    if (n_tr > MAX_TRUNS) n_tr = MAX_TRUNS;
+    {
+        int tot_it;
+        (void)block_exclusive_scan<RUN_THREADS>(n_it, sm.ws, tot_it);
+        n_it = tot_it;
     }
     // the item list slot is claimed now and used at the end, so the atomic's
     // latency overlaps the table work
@@ -733,29 +944,20 @@ __global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, in
             }
             if (t == 0) {
                 sm.tr_flat[n_tr] = n_flat;
-                // greedy groups of consecutive table runs that fit TAB_WORDS
-                int g = 0, used = 0, j = 0, e = 0, gx = 0;
+                // greedy groups of consecutive table runs that fit one buffer
+                int g = 0, used = 0, gx = 0;
                 sm.g_first[0] = 0;
                 for (int tr = 0; tr < n_tr; ++tr) {
-                    const int np = sm.tr_np[tr];
-                    const int words = 16 * np * (4 + sm.tr_rw[tr]);
+                    const int words = sm.tr_words[tr];
                     if (used + words > TAB_WORDS) {
-                        sm.g_j[g] = j;
-                        sm.g_e[g] = e;
                         sm.g_xw[g] = (uint8_t)gx;
                         sm.g_first[++g] = tr;
-                        used = j = e = gx = 0;
+                        used = gx = 0;
                     }
                     gx = gx > sm.tr_xw[tr] ? gx : sm.tr_xw[tr];
                     sm.tr_tab[tr] = used;
-                    sm.tr_j0[tr] = j;
-                    sm.tr_e0[tr] = e;
                     used += words;
-                    j += 4 * np;
-                    e += 16 * np;
                 }
-                sm.g_j[g] = j;
-                sm.g_e[g] = e;
                 sm.g_xw[g] = (uint8_t)gx;
                 sm.g_first[++g] = n_tr;
                 sm.n_groups = g;
@@ -764,80 +966,64 @@ __global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, in
         __syncthreads();
 
         const int n_groups = sm.n_groups;
+        // thread 0 copies the tables of group g into buffer g & 1
+        auto issue = [&](int g) {
+            const int ga = sm.g_first[g], gb = sm.g_first[g + 1];
+            uint32_t bytes = 0;
+            for (int tr = ga; tr < gb; ++tr) bytes += 4u * (uint32_t)sm.tr_words[tr];
+            unsigned long long* bar = &sm.bar[g & 1];
+            uint32_t* buf = reinterpret_cast<uint32_t*>(sm.table[g & 1]);
+            const unsigned long long keep = l2_policy_evict_last();  // tables are read by many CTAs
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(bar, bytes);
+            for (int tr = ga; tr < gb; ++tr)
+                bulk_copy_g2s_hint(buf + sm.tr_tab[tr], pool + sm.tr_src[tr], 4u * (uint32_t)sm.tr_words[tr], bar,
+                                   keep);
+        };
+        if (t == 0) issue(0);
+        // the first feature words of every table query, beside the copies
+        {
+            const int n_flat = sm.tr_flat[n_tr];
+            uint32_t* xsw = reinterpret_cast<uint32_t*>(sm.xs);
+            for (int f = t; f < n_flat; f += RUN_THREADS) {
+                const uint32_t fv = sm.flat[f];
+                const int64_t i = (int64_t)sm.idx[fv & 0xFFFFu];
+                const uint32_t* src = x + i * stride;
+                if (xvec) {
+                    cp_async16(sm.xs + f, src);  // stride >= 4 words: inside the row
+                } else {
+                    const int xw = sm.tr_xw[fv >> 16];
+                    for (int v = 0; v < XS_WORDS && v < xw; ++v) cp_async4(xsw + 4 * f + v, src + v);
+                }
+            }
+            cp_async_commit();
+        }
+        int fail_g = -1;
         for (int g = 0; g < n_groups; ++g) {
-            const int ga = sm.g_first[g], gb = sm.g_first[g + 1] - 1;
-            // single-coordinate entries E_j (v = 1, 2, 4, 8) and the zero entry
-            for (int f = t; f < sm.g_j[g]; f += RUN_THREADS) {
-                const int tr = find_item(sm.tr_j0, ga, gb, f);
-                const int j = f - sm.tr_j0[tr];
-                const int np = sm.tr_np[tr], rw = sm.tr_rw[tr];
-                CtxDesc cd{};
-                cd.d = sm.tr_d[tr];
-                cd.wd = sm.tr_wd[tr];
-                cd.slot_off = sm.tr_slot_off[tr];
-                cd.xw_off = sm.tr_xw_off[tr];
-                cd.pw_off = sm.tr_pw_off[tr];
-                uint4 z;
-                uint32_t er[TAB_RW];
-                single_entry(s, cd, j, z, er);
-                uint32_t* tab = table + sm.tr_tab[tr];
-                uint2* Zl = reinterpret_cast<uint2*>(tab);
-                uint2* Zh = Zl + np * 16;
-                uint32_t* R = tab + 64 * np;
-                const int e = (j >> 2) * 16 + (1 << (j & 3));
-                Zl[e] = make_uint2(z.x, z.y);
-                Zh[e] = make_uint2(z.z, z.w);
-                for (int u = 0; u < rw; ++u) R[u * 16 * np + e] = er[u];
-                if ((j & 3) == 0) {
-                    const int e0 = (j >> 2) * 16;
-                    Zl[e0] = make_uint2(0, 0);
-                    Zh[e0] = make_uint2(0, 0);
-                    for (int u = 0; u < rw; ++u) R[u * 16 * np + e0] = 0;
-                }
-            }
+            if (t == 0 && g + 1 < n_groups) issue(g + 1);
+            if (g == 0) cp_async_wait_all();
+            const bool ok = mbar_wait_bounded(&sm.bar[g & 1], (uint32_t)((g >> 1) & 1));
+            if (!ok) sm.failed = 1;
             __syncthreads();
-            // entries of two or more coordinates: XOR of their single entries
-            for (int f = t; f < sm.g_e[g]; f += RUN_THREADS) {
-                const int v = f & 15;
-                if (__popc(v) < 2) continue;
-                const int tr = find_item(sm.tr_e0, ga, gb, f);
-                const int e = f - sm.tr_e0[tr];
-                const int np = sm.tr_np[tr], rw = sm.tr_rw[tr];
-                uint32_t* tab = table + sm.tr_tab[tr];
-                uint2* Zl = reinterpret_cast<uint2*>(tab);
-                uint2* Zh = Zl + np * 16;
-                uint32_t* R = tab + 64 * np;
-                const int eb = e & ~15;
-                uint2 lo = make_uint2(0, 0), hi = make_uint2(0, 0);
-                uint32_t rr[TAB_RW] = {0, 0, 0, 0};
-#pragma unroll
-                for (int bb = 0; bb < 4; ++bb) {
-                    if ((v >> bb) & 1) {
-                        const int es = eb + (1 << bb);
-                        const uint2 l = Zl[es], h = Zh[es];
-                        lo.x ^= l.x;
-                        lo.y ^= l.y;
-                        hi.x ^= h.x;
-                        hi.y ^= h.y;
-#pragma unroll
-                        for (int u = 0; u < TAB_RW; ++u)
-                            if (u < rw) rr[u] ^= R[u * 16 * np + es];
-                    }
-                }
-                Zl[e] = lo;
-                Zh[e] = hi;
-#pragma unroll
-                for (int u = 0; u < TAB_RW; ++u)
-                    if (u < rw) R[u * 16 * np + e] = rr[u];
+            if (sm.failed) {
+                fail_g = g;
+                break;
             }
-            __syncthreads();
-            // the queries of the group's runs
-            const int fa = sm.tr_flat[ga], fb = sm.tr_flat[gb + 1];
+            const uint32_t* table = reinterpret_cast<const uint32_t*>(sm.table[g & 1]);
+            const int fa = sm.tr_flat[sm.g_first[g]], fb = sm.tr_flat[sm.g_first[g + 1]];
             if (sm.g_xw[g] <= 4)
-                query_group<5, 4, 3>(s, sm, table, x, stride, xvec, y, in_span, fa, fb);
+                query_group<5>(s, sm, table, x, stride, y, in_span, fa, fb);
             else
-                query_group<TAB_WD, TAB_WD, 1>(s, sm, table, x, stride, xvec, y, in_span, fa, fb);
+                query_group<TAB_WD>(s, sm, table, x, stride, y, in_span, fa, fb);
             __syncthreads();
+        }
+        if (fail_g >= 0) {
+            // a copy did not complete in time: record it, then let the copies
+            // still in flight land before the CTA's shared memory is released
+            if (t == 0) record_status(s.status, F2_ERR_TIMEOUT);
+            for (int g = fail_g; g < n_groups && g <= fail_g + 1; ++g)
+                (void)mbar_wait_bounded(&sm.bar[g & 1], (uint32_t)((g >> 1) & 1));
+            return;
         }
     }
 
@@ -853,7 +1039,7 @@ __global__ void __launch_bounds__(RUN_THREADS, 2) enc_runs_kernel(StoreDev s, in
         if (rr < n_runs && sm.run_tr[rr] < 0) {
             a = sm.starts[rr];
             b = sm.starts[rr + 1];
-            c = (uint32_t)(sm.ent[a] >> 32);
+            c = (uint32_t)(__ldg(sorted + seg0 + a) >> 32);
         }
         int tot;
         int it = it0 + block_exclusive_scan<RUN_THREADS>((b - a + ITEM_MAX - 1) / ITEM_MAX, sm.ws, tot);
@@ -877,6 +1063,12 @@ struct ShortSmem {
     int32_t pbase[SHORT_WARPS][TAB_WD + 1];
 };
 
+// A warp per item (round robin over a grid of one resident wave).  The loads
+// that do not depend on an item's basis (the item, its queries, the
+// context's descriptor, rank and pivot words) run one item ahead; the basis
+// rows themselves are fetched by asynchronous copies issued together, with
+// the query's feature words and the next item's pivot words in flight
+// beside them.
 __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
                                                                   const unsigned long long* __restrict__ sorted,
                                                                   const uint32_t* __restrict__ x, int stride,
@@ -894,9 +1086,7 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
     const int total = *n_items;
     const int nwarps = gridDim.x * SHORT_WARPS;
     const bool xvec = ((uintptr_t)x % 16) == 0 && (stride % 4) == 0;
-    // An item is (position | (length - 1) << 25, context).  The loads of an
-    // item that do not depend on its basis (the item, its queries' ids, the
-    // context's descriptor and rank) are issued one item ahead.
+    // An item is (position | (length - 1) << 25, context).
     auto unpack = [&](unsigned long long it, int& pos, int& len, int32_t& c) {
         pos = (int)(it & ((1u << ITEM_POS_BITS) - 1u));
         len = (int)((it >> ITEM_POS_BITS) & 31u) + 1;
@@ -904,10 +1094,9 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
     };
     int itx = blockIdx.x * SHORT_WARPS + wid;
     if (itx >= total) return;
-    unsigned long long item = __ldg(items + itx);
     int pos, len;
     int32_t c;
-    unpack(item, pos, len, c);
+    unpack(__ldg(items + itx), pos, len, c);
     unsigned long long en = __ldg(sorted + pos + (lane < len ? lane : 0));
     CtxDesc cd{};
     int rank = 0;
@@ -915,20 +1104,32 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
         cd = s.desc[c];
         rank = s.rank[c];
     }
+    uint32_t pw = (c < s.num_ctx && lane < cd.wd) ? __ldg(s.pivot + cd.pw_off + lane) : 0u;
+    unsigned long long item_n = (itx + nwarps < total) ? __ldg(items + itx + nwarps) : 0ull;
     while (true) {
-        const int64_t i = (int64_t)(uint32_t)en;
         const int nxt = itx + nwarps;
-        const unsigned long long item_n = (nxt < total) ? __ldg(items + nxt) : 0ull;
-        const int rs = (4 + cd.wd + 3) & ~3;  // staged row stride, 16-byte aligned
+        // the next item's queries, descriptor and rank (its item word is in)
+        int pos_n = 0, len_n = 1;
+        int32_t c_n = s.num_ctx;
+        unsigned long long en_n = 0;
+        CtxDesc cd_n{};
+        int rank_n = 0;
+        if (nxt < total) {
+            unpack(item_n, pos_n, len_n, c_n);
+            en_n = __ldg(sorted + pos_n + (lane < len_n ? lane : 0));
+            if (c_n < s.num_ctx) {
+                cd_n = s.desc[c_n];
+                rank_n = s.rank[c_n];
+            }
+        }
+        const unsigned long long item_nn = (nxt + nwarps < total) ? __ldg(items + nxt + nwarps) : 0ull;
+
+        const int64_t i = (int64_t)(uint32_t)en;
+        const int rs = row_stride(cd.wd);  // staged row: [z_k | r_k], 16-byte aligned
         const bool staged = c < s.num_ctx && cd.wd <= TAB_WD && cd.xw <= stride && rank * rs <= SHORT_REGION;
-        uint4 acc = make_uint4(0, 0, 0, 0);
-        bool ok = false;
+        uint32_t xr[TAB_WD];
         if (staged) {
-            // feature words and pivot words together
-            uint32_t xr[TAB_WD];
-            load_x<TAB_WD>(x + i * stride, lane < len ? cd.xw : 0, xvec, xr);
-            const uint32_t pw = (lane < cd.wd) ? __ldg(s.pivot + cd.pw_off + lane) : 0u;
-            // pivot list, word by word, and the staged rows [z_k | r_k]
+            // pivot list, word by word
             const int cnt = __popc(pw);
             int inc = cnt;
 #pragma unroll
@@ -946,20 +1147,33 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
                 }
             }
             __syncwarp();
+            // the pivot rows: z_k by one 16-byte copy, r_k word by word
+            for (int idx = lane; idx < rank; idx += 32)
+                cp_async16(region + idx * rs, s.bz + cd.slot_off + piv[idx]);
             {
-                const int cols = 4 + cd.wd;
-                const int per = 32 / cols;
-                const int row_in = lane / cols, col = lane - row_in * cols;
-                if (row_in < per) {
-                    for (int idx = row_in; idx < rank; idx += per) {
-                        const int k = piv[idx];
-                        const uint32_t v =
-                            (col < 4) ? __ldg(reinterpret_cast<const uint32_t*>(s.bz + cd.slot_off + k) + col)
-                                      : __ldg(s.bx + cd.xw_off + (int64_t)k * cd.wd + (col - 4));
-                        region[idx * rs + col] = v;
+                const int wd = cd.wd;
+                int idx = lane / wd, v = lane - (lane / wd) * wd;
+                const int di = 32 / wd, dv = 32 - di * wd;
+                for (int u = lane; u < rank * wd; u += 32) {
+                    cp_async4(region + idx * rs + 4 + v, s.bx + cd.xw_off + (int64_t)piv[idx] * wd + v);
+                    idx += di;
+                    v += dv;
+                    if (v >= wd) {
+                        v -= wd;
+                        ++idx;
                     }
                 }
             }
+            cp_async_commit();
+            load_x<TAB_WD>(x + i * stride, lane < len ? cd.xw : 0, xvec, xr);
+        }
+        // the next item's pivot words, beside this item's copies
+        const uint32_t pw_n =
+            (nxt < total && c_n < s.num_ctx && lane < cd_n.wd) ? __ldg(s.pivot + cd_n.pw_off + lane) : 0u;
+        uint4 acc = make_uint4(0, 0, 0, 0);
+        bool ok = false;
+        if (staged) {
+            cp_async_wait_all();
             __syncwarp();
             uint32_t q[TAB_WD];
             make_q<TAB_WD>(s.raw != 0, cd.n, xr, q);
@@ -995,20 +1209,6 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
             for (int v = 0; v < TAB_WD; ++v) resid |= q[v];
             ok = resid == 0;
         }
-        // the next item's query ids, descriptor and rank
-        int pos_n = 0, len_n = 1;
-        int32_t c_n = s.num_ctx;
-        unsigned long long en_n = 0;
-        CtxDesc cd_n{};
-        int rank_n = 0;
-        if (nxt < total) {
-            unpack(item_n, pos_n, len_n, c_n);
-            en_n = __ldg(sorted + pos_n + (lane < len_n ? lane : 0));
-            if (c_n < s.num_ctx) {
-                cd_n = s.desc[c_n];
-                rank_n = s.rank[c_n];
-            }
-        }
         if (lane < len) {
             if (staged) {
                 y[i] = ok ? acc : make_uint4(0, 0, 0, 0);
@@ -1018,7 +1218,7 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
             }
         }
         if (nxt >= total) break;
-        __syncwarp();  // the region is rewritten by the next item
+        __syncwarp();  // the region and pivot list are rewritten by the next item
         itx = nxt;
         pos = pos_n;
         len = len_n;
@@ -1026,6 +1226,8 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
         en = en_n;
         cd = cd_n;
         rank = rank_n;
+        pw = pw_n;
+        item_n = item_nn;
     }
 }
 
@@ -1041,11 +1243,17 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         return F2_ERR_ALIGN;
     cudaStream_t cs = (cudaStream_t)stream;
     const int64_t sub = Q < ENC_SUB ? Q : ENC_SUB;
-    const int64_t N = (int64_t)st->num_ctx + 1;  // buckets (the last for bad ids)
-    const int64_t T = (N + SCAN_TILE - 1) / SCAN_TILE;
-    // bucket scratch (32-bit words): sizes / starts [N], tile sums and
-    // prefixes [T], ticket, item count
-    const int64_t bin_words = N + 2 * T + 2;
+    int shift = st->enc_chunk_shift;
+    while ((sub >> shift) >= ENC_MAX_CHUNKS) ++shift;
+    const int64_t nch_max = (sub + (int64_t(1) << shift) - 1) >> shift;
+    const int64_t B = (int64_t)st->num_ctx + 1;  // buckets per chunk (the last for bad ids)
+    // 32-bit scratch: chunk counts [nch*B], scan input / starts [(nch+1)*B],
+    // scan tile sums and prefixes [T each], ticket, item count
+    const int64_t scan_n = (nch_max + 1) * B;
+    const int64_t T = (scan_n + SCAN_TILE - 1) / SCAN_TILE;
+    // + the table-build work list [9B] and its count, an aligned 8-byte pool counter
+    const int64_t bin_words = nch_max * B + scan_n + 2 * T + 2 + 9 * B + 1 + 4;
+    const bool tables = st->enc_table_min <= sub && st->num_ctx < (1 << 27);  // work items pack (context, block)
     cudaError_t e = cudaSuccess;
     // scratch, grown stream-ordered and kept by the store
     if (sub > st->enc_q_cap) {
@@ -1070,6 +1278,35 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
             return F2_ERR_OOM;
         st->enc_bin_cap = bin_words;
     }
+    if (B > st->enc_meta_cap) {
+        if (st->enc_hot) cudaFreeAsync(st->enc_hot, cs);
+        if (st->enc_tab_off) cudaFreeAsync(st->enc_tab_off, cs);
+        st->enc_hot = nullptr;
+        st->enc_tab_off = nullptr;
+        st->enc_meta_cap = 0;
+        e = cudaMallocAsync((void**)&st->enc_hot, (size_t)B, cs);
+        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->enc_tab_off, sizeof(long long) * (size_t)B, cs);
+        if (e != cudaSuccess) return F2_ERR_OOM;
+        st->enc_meta_cap = B;
+    }
+    if (tables && !st->enc_pool) {
+        // room for the table of every context that can have one (a table
+        // never outgrows its upper bound for rank 0), capped
+        int64_t words = 0;
+        for (int32_t c = 0; c < st->num_ctx; ++c) {
+            const int d = (st->flags & F2_FLAG_RAW_FEATURES) ? st->n_bits[c] : st->n_bits[c] + 1;
+            if ((d + 31) / 32 <= TAB_WD) {
+                const int wmax = 16 * ((d + 3) / 4) * (4 + ((d + 31) / 32 < TAB_RW ? (d + 31) / 32 : TAB_RW));
+                words += wmax < TAB_WORDS ? wmax : TAB_WORDS;
+            }
+        }
+        if (words > POOL_MAX_WORDS) words = POOL_MAX_WORDS;
+        if (words > 0) {
+            if (cudaMallocAsync((void**)&st->enc_pool, sizeof(uint32_t) * (size_t)words, cs) != cudaSuccess)
+                return F2_ERR_OOM;
+            st->enc_pool_words = words;
+        }
+    }
     e = cudaFuncSetAttribute(enc_runs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RunSmem));
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(enc_short_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1083,27 +1320,64 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         st->enc_short_per_sm = per > 0 ? per : 1;
     }
     const int short_per_sm = st->enc_short_per_sm;
-    int32_t* bins = st->enc_bins;
-    int32_t* tsum = bins + N;
+    if (tables) {
+        const int rc = f2_ensure_aux(st);
+        if (rc != F2_OK) return rc;
+    }
+    int32_t* cnt = st->enc_bins;
+    int32_t* sta = cnt + nch_max * B;
+    int32_t* tsum = sta + scan_n;
     int32_t* tpre = tsum + T;
     int32_t* ticket = tpre + T;
     int32_t* n_items = ticket + 1;
+    int32_t* hot_list = n_items + 1;
+    int32_t* n_hot = hot_list + 9 * B;
+    unsigned long long* pool_used = reinterpret_cast<unsigned long long*>(
+        (reinterpret_cast<uintptr_t>(n_hot + 1) + 7) & ~uintptr_t(7));
     unsigned long long* items = st->enc_items;
     const StoreDev sd = st->dev();
+    const int tbl_blocks = (int)((B + TBL_THREADS - 1) / TBL_THREADS);
     for (int64_t q0 = 0; q0 < Q; q0 += sub) {
         const int32_t n = (int32_t)((Q - q0) < sub ? (Q - q0) : sub);
+        const int32_t nch = (int32_t)((n + (int64_t(1) << shift) - 1) >> shift);
+        const int64_t sn = ((int64_t)nch + 1) * B;
+        const int32_t Tn = (int32_t)((sn + SCAN_TILE - 1) / SCAN_TILE);
         const uint32_t* xq = x + q0 * x_stride_words;
         uint4* yq = reinterpret_cast<uint4*>(y_out) + q0;
-        e = cudaMemsetAsync(bins, 0, sizeof(int32_t) * (size_t)N, cs);
+        e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * (size_t)(nch * B), cs);
         if (e == cudaSuccess) e = cudaMemsetAsync(ticket, 0, 2 * sizeof(int32_t), cs);
+        if (e == cudaSuccess) e = cudaMemsetAsync(n_hot, 0, sizeof(int32_t), cs);
+        if (e == cudaSuccess) e = cudaMemsetAsync(pool_used, 0, sizeof(unsigned long long), cs);
         if (e != cudaSuccess) return f2_cuda_status(e);
         enc_count_kernel<<<(n + ENC_TILE - 1) / ENC_TILE, ENC_TILE_THREADS, 0, cs>>>(n, ctx_id + q0, st->num_ctx,
-                                                                                   bins, st->enc_off);
-        enc_scan_kernel<<<(int)T, SCAN_THREADS, 0, cs>>>(bins, (int32_t)N, tsum, tpre, ticket);
+                                                                                   shift, (int32_t)B, cnt,
+                                                                                   st->enc_off);
+        enc_table_kernel<<<tbl_blocks, TBL_THREADS, 0, cs>>>(
+            sd, nch, (int32_t)B, cnt, sta, st->enc_hot, st->enc_tab_off, tables ? (long long)st->enc_pool_words : 0,
+            pool_used, hot_list, n_hot, tables ? st->enc_table_min : INT_MAX, (long long)st->enc_chunk_min,
+            x_stride_words);
+        // the tables are built on the second stream while the queries are
+        // placed (scan, scatter) on the caller's
+        if (tables) {
+            e = cudaEventRecord(st->ev_fork, cs);
+            if (e == cudaSuccess) e = cudaStreamWaitEvent(st->aux, st->ev_fork, 0);
+            if (e != cudaSuccess) return f2_cuda_status(e);
+            enc_build_kernel<<<st->num_sms * 8, TBL_THREADS, 0, st->aux>>>(sd, hot_list, n_hot, st->enc_tab_off,
+                                                                          st->enc_pool);
+            e = cudaEventRecord(st->ev_join, st->aux);
+            if (e != cudaSuccess) return f2_cuda_status(e);
+        }
+        enc_scan_kernel<<<Tn, SCAN_THREADS, 0, cs>>>(sta, (int32_t)sn, tsum, tpre, ticket);
         enc_scatter_kernel<<<(n + SCAT_THREADS * SCAT_PER - 1) / (SCAT_THREADS * SCAT_PER), SCAT_THREADS, 0, cs>>>(
-            n, ctx_id + q0, st->num_ctx, bins, tpre, st->enc_off, st->enc_sorted);
+            n, ctx_id + q0, st->num_ctx, shift, nch, (int32_t)B, cnt, sta, tpre, st->enc_hot, st->enc_off,
+            st->enc_sorted);
+        if (tables) {
+            e = cudaStreamWaitEvent(cs, st->ev_join, 0);
+            if (e != cudaSuccess) return f2_cuda_status(e);
+        }
         enc_runs_kernel<<<(n + RUN_SEG - 1) / RUN_SEG, RUN_THREADS, sizeof(RunSmem), cs>>>(
-            sd, n, st->enc_sorted, xq, x_stride_words, yq, in_span + q0, st->enc_table_min, items, n_items);
+            sd, n, st->enc_sorted, xq, x_stride_words, yq, in_span + q0, st->enc_hot, st->enc_tab_off,
+            st->enc_pool, items, n_items);
         enc_short_kernel<<<st->num_sms * short_per_sm, SHORT_THREADS, sizeof(ShortSmem), cs>>>(
             sd, st->enc_sorted, xq, x_stride_words, yq, in_span + q0, items, n_items);
         e = cudaGetLastError();
@@ -1166,4 +1440,6 @@ extern "C" int f2_encode_epilogue(const f2_store* st, int64_t Q, const int32_t* 
 }
 
 int f2_encode_table_min_default() { return DEFAULT_TABLE_MIN; }
-int f2_encode_table_min_floor() { return RUN_SEG / MAX_TRUNS; }
+int f2_encode_table_min_floor() { return 1; }
+int f2_encode_chunk_shift_default() { return DEFAULT_CHUNK_SHIFT; }
+long long f2_encode_chunk_min_default() { return DEFAULT_CHUNK_MIN; }

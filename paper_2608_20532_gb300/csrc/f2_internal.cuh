@@ -99,6 +99,112 @@ __device__ __forceinline__ void record_status(int* status, int code)
     atomicCAS(status, 0, code);
 }
 
+// ---------------------------------------------------------------------------
+// Asynchronous copies into shared memory (sm_90+ PTX): the 1-D bulk copy of
+// the tensor-memory-access unit, completed on an mbarrier by transaction
+// bytes, and the per-thread cp.async of 4/8/16 bytes.  Every wait is bounded
+// by a %globaltimer deadline; a wait that runs out returns false and the
+// caller records F2_ERR_TIMEOUT instead of hanging.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+// Make initialised mbarriers visible to the asynchronous proxy.
+__device__ __forceinline__ void mbar_init_fence() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+
+// Order this thread's earlier shared-memory accesses (generic proxy) before
+// later asynchronous-proxy writes to the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(unsigned long long* bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+}
+
+// dst (shared) and src (global) 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes, unsigned long long* bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_addr(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+
+// The same copy with an L2 cache-policy hint (a policy from l2_policy_*).
+__device__ __forceinline__ void bulk_copy_g2s_hint(void* dst, const void* src, uint32_t bytes, unsigned long long* bar,
+                                                   unsigned long long policy)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(policy)
+        : "memory");
+}
+
+// L2 policy: keep the lines (evict last), for data read again soon.
+__device__ __forceinline__ unsigned long long l2_policy_evict_last()
+{
+    unsigned long long p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ bool mbar_try_wait(unsigned long long* bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ unsigned long long global_ns()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+constexpr unsigned long long WAIT_LIMIT_NS = 200000000ull;  // 0.2 s: far above any copy's latency
+
+// Wait for the phase of `bar` with the given parity to complete, at most
+// WAIT_LIMIT_NS; false when the deadline passed first.
+__device__ __forceinline__ bool mbar_wait_bounded(unsigned long long* bar, uint32_t parity)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (global_ns() - t0 > WAIT_LIMIT_NS) return false;
+    return true;
+}
+
+// Per-thread asynchronous copies (cp.async, L1-allocating for 4/8 bytes,
+// L2-only for 16); completed by cp_async_wait_all.
+__device__ __forceinline__ void cp_async4(void* dst, const void* src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async16(void* dst, const void* src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group()
+{
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 }  // namespace f2
 
 struct f2_store {
@@ -120,8 +226,8 @@ struct f2_store {
     f2::Widths widths;      // width classes of the contexts (computed on first use)
     // second stream of the learn launches (kernels of independent width
     // classes run side by side), its fork and join events; created on first use
-    cudaStream_t aux;
-    cudaEvent_t ev_fork, ev_join;
+    mutable cudaStream_t aux;
+    mutable cudaEvent_t ev_fork, ev_join;
     bool widths_ready;
     std::vector<int32_t> n_bits;
     std::vector<int64_t> slot_off, xw_off, pw_off;
@@ -160,7 +266,15 @@ struct f2_store {
     mutable unsigned long long* enc_items;  // runs left to the per-warp kernel
     mutable int64_t enc_q_cap;
     mutable int enc_short_per_sm;           // resident CTAs of the per-warp encode kernel
-    int enc_table_min;                      // shortest run encoded with a table
+    mutable int enc_runs_per_sm;            // resident CTAs of the table encode kernel
+    int enc_table_min;                      // fewest queries of a context (per pass) that get a table
+    int enc_chunk_shift;                    // log2 of the queries of one locality chunk
+    int64_t enc_chunk_min;                  // fewest queries of a context (per pass) laid out chunk by chunk
+    mutable uint8_t* enc_hot;               // per bucket: encoded with a table in this pass
+    mutable long long* enc_tab_off;         // per bucket: word offset of its table in the pool
+    mutable uint32_t* enc_pool;             // lookup tables of the contexts with many queries
+    mutable int64_t enc_pool_words;
+    mutable int64_t enc_meta_cap;           // buckets of enc_hot / enc_tab_off
     // host-input entry points (f2_learn_host, f2_encode_host)
     f2::HostIO* hio;
     int64_t host_chunk_bytes;               // bytes of rows (or queries) per copied chunk
@@ -189,5 +303,8 @@ constexpr int64_t DEFAULT_HOST_CHUNK_BYTES = int64_t(512) << 20;
 // Host helpers (store.cu, encode.cu, host_io.cu).
 void f2_host_io_free(f2_store* st);
 int f2_cuda_status(cudaError_t e);
+int f2_ensure_aux(const f2_store* st);  // second stream and fork/join events, created on first use
 int f2_encode_table_min_default();
 int f2_encode_table_min_floor();
+int f2_encode_chunk_shift_default();
+long long f2_encode_chunk_min_default();

@@ -1582,15 +1582,9 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         st->rep_capacity = total_rows;
     }
     const StoreDev sd = st->dev();
-    if (!st->aux) {  // on the store's device
-        int cur = -1;
-        e = cudaGetDevice(&cur);
-        if (e == cudaSuccess && cur != st->device) e = cudaSetDevice(st->device);
-        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
-        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_fork, cudaEventDisableTiming);
-        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_join, cudaEventDisableTiming);
-        if (cur >= 0 && cur != st->device) cudaSetDevice(cur);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+    {
+        const int rc = f2_ensure_aux(st);
+        if (rc != F2_OK) return rc;
     }
     Fork fk{cs, st->aux, st->ev_fork, st->ev_join};
     if (dedup) {

@@ -17,6 +17,19 @@ int f2_cuda_status(cudaError_t e)
 
 static inline bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
+int f2_ensure_aux(const f2_store* st)
+{
+    if (st->aux) return F2_OK;
+    int cur = -1;  // created on the store's device
+    cudaError_t e = cudaGetDevice(&cur);
+    if (e == cudaSuccess && cur != st->device) e = cudaSetDevice(st->device);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_join, cudaEventDisableTiming);
+    if (cur >= 0 && cur != st->device) cudaSetDevice(cur);
+    return f2_cuda_status(e);
+}
+
 extern "C" const char* f2_status_string(int status)
 {
     switch (status) {
@@ -45,7 +58,8 @@ static void free_store(f2_store* s)
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
                     s->full_ctr, s->full_cnt, s->full_first,
-                    s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items};
+                    s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items, s->enc_hot, s->enc_tab_off,
+                    s->enc_pool};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     delete s;
@@ -88,6 +102,8 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->warp_work = DEFAULT_WARP_WORK;
     s->dedup = 1;
     s->enc_table_min = f2_encode_table_min_default();
+    s->enc_chunk_shift = f2_encode_chunk_shift_default();
+    s->enc_chunk_min = f2_encode_chunk_min_default();
     s->host_chunk_bytes = DEFAULT_HOST_CHUNK_BYTES;
     if (cudaGetDevice(&s->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
@@ -385,6 +401,14 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_ENCODE_TABLE_MIN:
         if (value < f2_encode_table_min_floor() || value > (int64_t(1) << 30)) return F2_ERR_INVALID_ARG;
         s->enc_table_min = (int)value;
+        return F2_OK;
+    case F2_OPT_ENCODE_CHUNK_SHIFT:
+        if (value < 11 || value > 25) return F2_ERR_INVALID_ARG;
+        s->enc_chunk_shift = (int)value;
+        return F2_OK;
+    case F2_OPT_ENCODE_CHUNK_MIN:
+        if (value < 1) return F2_ERR_INVALID_ARG;
+        s->enc_chunk_min = value;
         return F2_OK;
     case F2_OPT_HOST_CHUNK_BYTES:
         if (value < (int64_t(1) << 16)) return F2_ERR_INVALID_ARG;
