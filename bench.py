@@ -111,6 +111,98 @@ class ClockSampler:
                 "samples": len(inside)}
 
 
+class NvmlSampler:
+    """SM clock, power and clock-event reasons read through NVML (read-only
+    queries, ctypes) every few milliseconds while the timed region runs, so
+    that a region of a few tens of milliseconds still holds several samples.
+    Falls back to ClockSampler (nvidia-smi) where NVML cannot be loaded."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+               0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, device_index: int, period_s: float = 0.005):
+        import ctypes
+
+        self.samples = []
+        self.ok = False
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            bus = None
+            try:
+                import torch
+
+                pr = torch.cuda.get_device_properties(device_index)
+                bus = f"{pr.pci_domain_id:08x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0".encode()
+            except Exception:
+                bus = None
+            rc = lib.nvmlDeviceGetHandleByPciBusId_v2(bus, ctypes.byref(h)) if bus else 1
+            if rc != 0 and lib.nvmlDeviceGetHandleByIndex_v2(device_index, ctypes.byref(h)) != 0:
+                return
+            self.lib, self.h, self.ct = lib, h, ctypes
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or getattr(
+                lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            mx = ctypes.c_uint(0)
+            lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx))  # NVML_CLOCK_SM
+            self.max_mhz = float(mx.value) or None
+        except (OSError, AttributeError):
+            return
+        self.ok = True
+        self.period = period_s
+        self.stop_flag = False
+        self.t = threading.Thread(target=self._run, daemon=True)
+        self.t.start()
+
+    def _run(self):
+        ct, lib, h = self.ct, self.lib, self.h
+        clk, pw, rs = ct.c_uint(0), ct.c_uint(0), ct.c_ulonglong(0)
+        while not self.stop_flag:
+            lib.nvmlDeviceGetClockInfo(h, 1, ct.byref(clk))
+            lib.nvmlDeviceGetPowerUsage(h, ct.byref(pw))
+            self.reasons_fn(h, ct.byref(rs))
+            self.samples.append((time.time(), float(clk.value), pw.value / 1000.0, int(rs.value)))
+            time.sleep(self.period)
+
+    def stop(self, t0: float, t1: float) -> dict:
+        self.stop_flag = True
+        self.t.join(timeout=2)
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["no samples"], "samples": 0,
+                    "source": "nvml"}
+        reasons = sorted({name for _, _, _, r in inside for bit, name in self.REASONS.items() if r & bit})
+        return {"sm_mhz": statistics.median([c for _, c, _, _ in inside]), "sm_max_mhz": self.max_mhz,
+                "power_w_max": max(p for _, _, p, _ in inside), "reasons": reasons, "samples": len(inside),
+                "source": "nvml, 5 ms period"}
+
+
+def clock_sampler(device_index: int):
+    s = NvmlSampler(device_index)
+    return s if s.ok else ClockSampler(device_index)
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+
+    return platform.processor() or platform.machine()
+
+
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -306,7 +398,7 @@ def run_ours(args):
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(nev)] for _ in range(K)]
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(local)
+    sampler = clock_sampler(local)
     time.sleep(0.3)
     if world > 1:
         torch.distributed.barrier()
@@ -329,6 +421,7 @@ def run_ours(args):
     learn_ms = [e[0].elapsed_time(e[1]) for e in events]
     solve_ms = [e[1].elapsed_time(e[2]) for e in events]
     enc_ms = [e[2].elapsed_time(e[3]) for e in events]
+    each_ms = [e[0].elapsed_time(e[3]) for e in events]  # one step, bracketed by its own events
     total_ms = reduce_across_ranks(total_ms, "max", dev)
     ms_step = total_ms / K
 
@@ -516,6 +609,10 @@ def run_ours(args):
         "config": dict(describe(cfg_id, wl), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
         "phases_ms": {"learn": statistics.mean(learn_ms), "solve": statistics.mean(solve_ms),
                       "encode": statistics.mean(enc_ms)},
+        "step_stats_ms": {"mean": statistics.mean(each_ms), "median": statistics.median(each_ms),
+                          "best": min(each_ms),
+                          "learn": {"median": statistics.median(learn_ms), "best": min(learn_ms)},
+                          "encode": {"median": statistics.median(enc_ms), "best": min(enc_ms)}},
         "learn_rows_per_s": wl.total_rows / learn_mean,
         "roofline": roofline,
         "roofline_learn": rl_learn,
@@ -680,9 +777,16 @@ def cpu_baseline(wl, seconds: float) -> dict:
     qsel = _queries_for(wl, ctxs, frac)
     t = _oracle_step(_subset(wl, ctxs, qsel), threads)
     rows = int(wl.rows[ctxs].sum())
-    return {"value": rows / t, "unit": "rows/s", "cores": threads, "kind": "oracle",
+    # one thread, on a sample a sixth the size (a few seconds)
+    ctx1 = _sample(wl, max(20_000, target // 6), seed=4)
+    frac1 = wl.rows[ctx1].sum() / wl.total_rows
+    t1 = _oracle_step(_subset(wl, ctx1, _queries_for(wl, ctx1, frac1)), 1)
+    rows1 = int(wl.rows[ctx1].sum())
+    return {"value": rows / t, "unit": "rows/s", "cores": threads, "kind": "oracle", "cpu_model": cpu_model(),
             "sample": f"{len(ctxs)} of {wl.num_ctx} contexts ({rows} rows, {0 if qsel is None else len(qsel)} "
-                      f"queries, {100 * frac:.1f}% of the step), learn + solve + encode, {t:.1f} s"}
+                      f"queries, {100 * frac:.1f}% of the step), learn + solve + encode, {t:.1f} s",
+            "single_thread": {"value": rows1 / t1, "unit": "rows/s", "cores": 1,
+                              "sample": f"{len(ctx1)} contexts ({rows1} rows), {t1:.1f} s"}}
 
 
 def run_reference(args):
@@ -710,7 +814,8 @@ def run_reference(args):
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded planted affine maps)",
            "config": describe(args.config, wl),
-           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": threads, "kind": "oracle", "sample": sample},
+           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": threads, "kind": "oracle", "sample": sample,
+                            "cpu_model": cpu_model()},
            "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
 

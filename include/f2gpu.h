@@ -295,8 +295,11 @@ enum f2_option {
     F2_OPT_ENCODE_CHUNK_SHIFT = 7, /* log2 of the consecutive queries whose table-encoded results are
                                     written together (L2 locality of f2_encode_batched's output);
                                     default 20, in [11, 25]; raised so a pass has at most 64 chunks */
-    F2_OPT_ENCODE_CHUNK_MIN = 8  /* fewest queries of one context (in a pass) for which its queries are
+    F2_OPT_ENCODE_CHUNK_MIN = 8, /* fewest queries of one context (in a pass) for which its queries are
                                     laid out chunk by chunk (the others keep one run); default 1024 */
+    F2_OPT_FAIL_ALLOC = 9        /* test hook: the device allocation made after `value` more successful
+                                    ones by calls on this store fails as if out of memory (the call
+                                    returns F2_ERR_OOM; the store stays usable); -1 (default) = off */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 
@@ -317,7 +320,10 @@ int f2_set_option(f2_store* store, int option, int64_t value);
  *
  *   num_ctx        in [0, F2_NOALLOC_MAX_CTX]; larger values are rejected
  *                  with F2_ERR_INVALID_ARG before anything is enqueued.
- *   n_bits_host    host int32[num_ctx], each in [1, 1024] (F2_ERR_NBITS).
+ *                  With num_ctx == 0 the call only sets *status_dev to F2_OK.
+ *   n_bits_host    host int32[num_ctx], each in [1, 1024] (F2_ERR_NBITS);
+ *                  copied during the call (through a library-owned host
+ *                  array), so it may be reused as soon as the call returns.
  *   flags          0 or F2_FLAG_RAW_FEATURES, as for f2_create.
  *   state (device, caller-owned, in/out, canonical layout of f2_get_basis;
  *          sizes from d_c = n_c + 1 (n_c for raw rows), Wd_c = ceil(d_c/32)):
@@ -332,12 +338,14 @@ int f2_set_option(f2_store* store, int option, int64_t value);
  *                  first device-detected error (F2_ERR_ROWS).
  *   row_off_dev, x_dev, x_off_dev, y_dev, total_rows, total_x_words: one
  *                  CSR batch, exactly as for f2_learn_batched.
- * The first call on a device (per process) looks up the device address of
- * the scratch array with cudaGetSymbolAddress; make that first call before
- * any stream capture.  Every call shares the one scratch array and
- * rewrites what it uses, so calls that overlap on the GPU (different
- * streams, or different host threads) race: serialize them.  Results are
- * bit-identical to f2_learn_batched on the same inputs.
+ * The first call on a device (per process) does a one-time set-up: it looks
+ * up the device address of the scratch array with cudaGetSymbolAddress and
+ * loads every kernel this entry point can launch (loading a kernel's code
+ * may itself allocate device memory, so only this first call may allocate);
+ * make that first call before any stream capture.  Every call shares the
+ * one scratch array and rewrites what it uses, so calls that overlap on the
+ * GPU (different streams, or different host threads) race: serialize them.
+ * Results are bit-identical to f2_learn_batched on the same inputs.
  * Errors: F2_ERR_INVALID_ARG, F2_ERR_NBITS, F2_ERR_ALIGN, F2_ERR_CUDA.
  */
 #define F2_NOALLOC_MAX_CTX 16384

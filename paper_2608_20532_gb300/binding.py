@@ -36,6 +36,7 @@ F2_OPT_ENCODE_TABLE_MIN = 5
 F2_OPT_HOST_CHUNK_BYTES = 6
 F2_OPT_ENCODE_CHUNK_SHIFT = 7
 F2_OPT_ENCODE_CHUNK_MIN = 8
+F2_OPT_FAIL_ALLOC = 9
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

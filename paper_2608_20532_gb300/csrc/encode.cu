@@ -1236,6 +1236,7 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
 extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* ctx_id, const uint32_t* x,
                                  int32_t x_stride_words, uint32_t* y_out, uint8_t* in_span, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_encode_batched");
     if (!st || Q < 0 || x_stride_words < 1) return F2_ERR_INVALID_ARG;
     if (Q == 0) return F2_OK;
     if (!ctx_id || !x || !y_out || !in_span) return F2_ERR_INVALID_ARG;
@@ -1264,9 +1265,11 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         st->enc_sorted = nullptr;
         st->enc_items = nullptr;
         st->enc_q_cap = 0;
-        e = cudaMallocAsync((void**)&st->enc_off, sizeof(int32_t) * (size_t)sub, cs);
-        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->enc_sorted, sizeof(unsigned long long) * (size_t)sub, cs);
-        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->enc_items, sizeof(unsigned long long) * (size_t)sub, cs);
+        e = f2_dev_alloc(st, (void**)&st->enc_off, sizeof(int32_t) * (size_t)sub, cs, true);
+        if (e == cudaSuccess)
+            e = f2_dev_alloc(st, (void**)&st->enc_sorted, sizeof(unsigned long long) * (size_t)sub, cs, true);
+        if (e == cudaSuccess)
+            e = f2_dev_alloc(st, (void**)&st->enc_items, sizeof(unsigned long long) * (size_t)sub, cs, true);
         if (e != cudaSuccess) return F2_ERR_OOM;
         st->enc_q_cap = sub;
     }
@@ -1274,7 +1277,7 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         if (st->enc_bins) cudaFreeAsync(st->enc_bins, cs);
         st->enc_bins = nullptr;
         st->enc_bin_cap = 0;
-        if (cudaMallocAsync((void**)&st->enc_bins, sizeof(int32_t) * (size_t)bin_words, cs) != cudaSuccess)
+        if (f2_dev_alloc(st, (void**)&st->enc_bins, sizeof(int32_t) * (size_t)bin_words, cs, true) != cudaSuccess)
             return F2_ERR_OOM;
         st->enc_bin_cap = bin_words;
     }
@@ -1284,8 +1287,9 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         st->enc_hot = nullptr;
         st->enc_tab_off = nullptr;
         st->enc_meta_cap = 0;
-        e = cudaMallocAsync((void**)&st->enc_hot, (size_t)B, cs);
-        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->enc_tab_off, sizeof(long long) * (size_t)B, cs);
+        e = f2_dev_alloc(st, (void**)&st->enc_hot, (size_t)B, cs, true);
+        if (e == cudaSuccess)
+            e = f2_dev_alloc(st, (void**)&st->enc_tab_off, sizeof(long long) * (size_t)B, cs, true);
         if (e != cudaSuccess) return F2_ERR_OOM;
         st->enc_meta_cap = B;
     }
@@ -1302,7 +1306,7 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         }
         if (words > POOL_MAX_WORDS) words = POOL_MAX_WORDS;
         if (words > 0) {
-            if (cudaMallocAsync((void**)&st->enc_pool, sizeof(uint32_t) * (size_t)words, cs) != cudaSuccess)
+            if (f2_dev_alloc(st, (void**)&st->enc_pool, sizeof(uint32_t) * (size_t)words, cs, true) != cudaSuccess)
                 return F2_ERR_OOM;
             st->enc_pool_words = words;
         }
@@ -1426,6 +1430,7 @@ extern "C" int f2_encode_epilogue(const f2_store* st, int64_t Q, const int32_t* 
                                   const uint32_t* sc, const uint32_t* state, const uint32_t* opaque_mask,
                                   uint32_t* y, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_encode_epilogue");
     if (!st || Q < 0) return F2_ERR_INVALID_ARG;
     if (Q == 0) return F2_OK;
     if (!y || !in_span || !ctx_id) return F2_ERR_INVALID_ARG;

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 
 #include <vector>
@@ -11,6 +12,16 @@
 namespace f2 {
 
 struct HostIO;  // copy streams, events and staging of the host-input entry points
+
+// An NVTX range over one API call (visible in Nsight timelines; costs a
+// function-pointer check when no tool is attached).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
+#define F2_NVTX_RANGE(name) ::f2::NvtxRange f2_nvtx_range_(name)
 
 constexpr unsigned FULL = 0xffffffffu;
 constexpr int MAX_N = 1024;          // feature bits per context
@@ -275,6 +286,9 @@ struct f2_store {
     mutable uint32_t* enc_pool;             // lookup tables of the contexts with many queries
     mutable int64_t enc_pool_words;
     mutable int64_t enc_meta_cap;           // buckets of enc_hot / enc_tab_off
+    // test hook (F2_OPT_FAIL_ALLOC): device allocations left before one is
+    // made to fail; -1 = off
+    mutable int64_t fail_alloc_in;
     // host-input entry points (f2_learn_host, f2_encode_host)
     f2::HostIO* hio;
     int64_t host_chunk_bytes;               // bytes of rows (or queries) per copied chunk
@@ -303,6 +317,10 @@ constexpr int64_t DEFAULT_HOST_CHUNK_BYTES = int64_t(512) << 20;
 // Host helpers (store.cu, encode.cu, host_io.cu).
 void f2_host_io_free(f2_store* st);
 int f2_cuda_status(cudaError_t e);
+// Every device allocation made by a call on a store goes through here (the
+// stream-ordered allocator with a stream, cudaMalloc without one), so the
+// F2_OPT_FAIL_ALLOC hook can make it fail.
+cudaError_t f2_dev_alloc(const f2_store* st, void** p, size_t bytes, cudaStream_t cs, bool stream_ordered);
 int f2_ensure_aux(const f2_store* st);  // second stream and fork/join events, created on first use
 int f2_encode_table_min_default();
 int f2_encode_table_min_floor();

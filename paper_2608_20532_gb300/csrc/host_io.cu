@@ -95,13 +95,13 @@ int host_io(f2_store* st, HostIO** out)
 
 // Grow a device buffer (contents are not kept); the caller has synchronized.
 template <typename T>
-cudaError_t grow(T*& p, int64_t& cap, int64_t need)
+cudaError_t grow(const f2_store* st, T*& p, int64_t& cap, int64_t need)
 {
     if (need <= cap) return cudaSuccess;
     if (p) cudaFree(p);
     p = nullptr;
     cap = 0;
-    const cudaError_t e = cudaMalloc((void**)&p, sizeof(T) * (size_t)(need > 0 ? need : 1));
+    const cudaError_t e = f2_dev_alloc(st, (void**)&p, sizeof(T) * (size_t)(need > 0 ? need : 1), nullptr, false);
     if (e == cudaSuccess) cap = need;
     return e;
 }
@@ -139,6 +139,7 @@ void f2_host_io_free(f2_store* st)
 extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_t* x, const int64_t* x_off,
                              const uint32_t* y, int64_t total_rows, int64_t total_x_words, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_learn_host");
     if (!st || total_rows < 0 || total_x_words < 0) return F2_ERR_INVALID_ARG;
     const int32_t C = st->num_ctx;
     if (C == 0) return F2_OK;
@@ -186,21 +187,25 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
         e = sync_all(h, cs);
         for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
             int64_t xc = h->x_cap, yc = h->y_cap, cc = h->c_cap, cc2 = h->c_cap;
-            e = grow(h->x[b], xc, need_x);
-            if (e == cudaSuccess) e = grow(h->y[b], yc, need_y);
-            if (e == cudaSuccess) e = grow(h->ro[b], cc, need_c);
-            if (e == cudaSuccess) e = grow(h->xo[b], cc2, need_c);
+            e = grow(st, h->x[b], xc, need_x);
+            if (e == cudaSuccess) e = grow(st, h->y[b], yc, need_y);
+            if (e == cudaSuccess) e = grow(st, h->ro[b], cc, need_c);
+            if (e == cudaSuccess) e = grow(st, h->xo[b], cc2, need_c);
         }
         if (e == cudaSuccess) {
             h->x_cap = std::max(h->x_cap, need_x);
             h->y_cap = std::max(h->y_cap, need_y);
             h->c_cap = std::max(h->c_cap, need_c);
             int64_t fc = h->full_cap, fc2 = h->full_cap;
-            e = grow(h->row_off, fc, (int64_t)C + 1);
-            if (e == cudaSuccess) e = grow(h->x_off, fc2, (int64_t)C + 1);
+            e = grow(st, h->row_off, fc, (int64_t)C + 1);
+            if (e == cudaSuccess) e = grow(st, h->x_off, fc2, (int64_t)C + 1);
             if (e == cudaSuccess) h->full_cap = std::max<int64_t>(h->full_cap, (int64_t)C + 1);
         }
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        if (e != cudaSuccess) {
+            // a buffer may have been freed: regrow every one on the next call
+            h->x_cap = h->y_cap = h->c_cap = h->full_cap = 0;
+            return f2_cuda_status(e);
+        }
     }
     for (size_t j = 0; j < chunks.size(); ++j) {
         const Chunk& k = chunks[j];
@@ -241,6 +246,7 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
 extern "C" int f2_encode_host(const f2_store* cst, int64_t Q, const int32_t* ctx_id, const uint32_t* x,
                               int32_t x_stride_words, uint32_t* y_out, uint8_t* in_span, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_encode_host");
     if (!cst || Q < 0 || x_stride_words < 1) return F2_ERR_INVALID_ARG;
     if (Q == 0) return F2_OK;
     if (!ctx_id || !x || !y_out || !in_span) return F2_ERR_INVALID_ARG;
@@ -262,12 +268,15 @@ extern "C" int f2_encode_host(const f2_store* cst, int64_t Q, const int32_t* ctx
         e = sync_all(h, cs);
         for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
             int64_t a = h->q_cap, a2 = h->q_cap, a3 = h->q_cap, ax = h->qx_cap;
-            e = grow(h->qc[b], a, qn);
-            if (e == cudaSuccess) e = grow(h->qy[b], a2, qn);
-            if (e == cudaSuccess) e = grow(h->qs[b], a3, qn);
-            if (e == cudaSuccess) e = grow(h->qx[b], ax, qn * x_stride_words);
+            e = grow(st, h->qc[b], a, qn);
+            if (e == cudaSuccess) e = grow(st, h->qy[b], a2, qn);
+            if (e == cudaSuccess) e = grow(st, h->qs[b], a3, qn);
+            if (e == cudaSuccess) e = grow(st, h->qx[b], ax, qn * x_stride_words);
         }
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        if (e != cudaSuccess) {
+            h->q_cap = h->qx_cap = 0;  // a buffer may have been freed: regrow every one next time
+            return f2_cuda_status(e);
+        }
         h->q_cap = std::max(h->q_cap, qn);
         h->qx_cap = std::max(h->qx_cap, qn * x_stride_words);
     }

@@ -36,6 +36,7 @@
 // by a separate wide kernel.  Single-block plan kernels validate the CSR
 // batch and order the work longest-first.
 #include <limits.h>
+#include <string.h>
 
 #include <mutex>
 
@@ -1563,6 +1564,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
                                 const uint32_t* y, int64_t total_rows, int64_t total_x_words,
                                 f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_learn_batched");
     if (!st || total_rows < 0 || total_x_words < 0) return F2_ERR_INVALID_ARG;
     if (st->num_ctx == 0) return F2_OK;
     if (!row_off || !x_off || (!x && total_x_words) || (!y && total_rows)) return F2_ERR_INVALID_ARG;
@@ -1576,9 +1578,9 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (st->rep_dup) cudaFreeAsync(st->rep_dup, cs);
         st->rep_list = st->rep_dup = nullptr;
         st->rep_capacity = 0;
-        e = cudaMallocAsync((void**)&st->rep_list, sizeof(int32_t) * (size_t)total_rows, cs);
-        if (e == cudaSuccess) e = cudaMallocAsync((void**)&st->rep_dup, sizeof(int32_t) * (size_t)total_rows, cs);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        e = f2_dev_alloc(st, (void**)&st->rep_list, sizeof(int32_t) * (size_t)total_rows, cs, true);
+        if (e == cudaSuccess) e = f2_dev_alloc(st, (void**)&st->rep_dup, sizeof(int32_t) * (size_t)total_rows, cs, true);
+        if (e != cudaSuccess) return F2_ERR_OOM;
         st->rep_capacity = total_rows;
     }
     const StoreDev sd = st->dev();
@@ -1691,30 +1693,6 @@ struct NoallocDevice {
 NoallocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
 std::mutex g_noalloc_mu;
 
-// Once per device (with that device current): resolve the scratch address.
-int noalloc_setup(NoallocDevice** out)
-{
-    int device = -1;
-    cudaError_t e = cudaGetDevice(&device);
-    if (e != cudaSuccess) return f2_cuda_status(e);
-    if (device < 0 || device >= NOALLOC_MAX_DEVICES) return F2_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    NoallocDevice& d = g_noalloc_dev[device];
-    if (!d.ready) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || p == nullptr) return e != cudaSuccess ? f2_cuda_status(e) : F2_ERR_CUDA;
-        int sms = 0;
-        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-        if (e != cudaSuccess) return f2_cuda_status(e);
-        d.scratch = static_cast<NoallocScratch*>(p);
-        d.num_sms = sms;
-        d.ready = true;
-    }
-    *out = &d;
-    return F2_OK;
-}
-
 // Context descriptors and canonical offsets (exclusive prefix sums of d,
 // d*wd and wd) for up to F2_NOALLOC_MAX_CTX contexts, one block.
 __global__ void __launch_bounds__(1024) noalloc_desc_kernel(const int32_t* __restrict__ n_bits, int C, uint32_t raw,
@@ -1790,6 +1768,55 @@ __global__ void __launch_bounds__(1024) noalloc_desc_kernel(const int32_t* __res
     }
 }
 
+// Host copy of the caller's widths: the device copy is made from here, so the
+// caller's array is free again when the call returns (a copy from pageable
+// memory is staged before cudaMemcpyAsync returns).  Guarded by g_noalloc_mu.
+int32_t g_noalloc_nbits[F2_NOALLOC_MAX_CTX];
+
+// Every kernel the allocation-free path can launch.  Loading a kernel's code
+// (on its first launch, under lazy module loading) may allocate device
+// memory, so the first call on a device loads all of them.
+cudaError_t noalloc_load_kernels()
+{
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, noalloc_desc_kernel);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_key_kernel);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_scan_kernel);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_scatter_kernel);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<true>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<false>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_wide_kernel<WIDE_WD, CLS_WIDE>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_wide_kernel<WIDE_M_WD, CLS_WIDE_M>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, verify_full_kernel);
+    return e;
+}
+
+// Once per device (with that device current): resolve the scratch address
+// and load the kernels.
+int noalloc_setup(NoallocDevice** out)
+{
+    int device = -1;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return f2_cuda_status(e);
+    if (device < 0 || device >= NOALLOC_MAX_DEVICES) return F2_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoallocDevice& d = g_noalloc_dev[device];
+    if (!d.ready) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || p == nullptr) return e != cudaSuccess ? f2_cuda_status(e) : F2_ERR_CUDA;
+        int sms = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+        if (e == cudaSuccess) e = noalloc_load_kernels();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        d.scratch = static_cast<NoallocScratch*>(p);
+        d.num_sms = sms;
+        d.ready = true;
+    }
+    *out = &d;
+    return F2_OK;
+}
+
 }  // namespace
 
 extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
@@ -1800,10 +1827,12 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
                                         const uint32_t* y_dev, int64_t total_rows, int64_t total_x_words,
                                         f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_learn_batched_noalloc");
     if (num_ctx < 0 || num_ctx > F2_NOALLOC_MAX_CTX || (flags & ~F2_FLAG_RAW_FEATURES) || total_rows < 0 ||
         total_x_words < 0 || !status_dev)
         return F2_ERR_INVALID_ARG;
-    if (num_ctx == 0) return F2_OK;
+    if (num_ctx == 0)  // nothing to learn: only the status word is written
+        return f2_cuda_status(cudaMemsetAsync(status_dev, 0, sizeof(int32_t), (cudaStream_t)stream));
     if (!n_bits_host || !rank_dev || !pivot_mask_dev || !basis_x_dev || !basis_z_dev || !contra_dev ||
         !first_contra_dev || !n_contra_dev || !rows_seen_dev || !row_off_dev || !x_off_dev ||
         (!x_dev && total_x_words) || (!y_dev && total_rows))
@@ -1823,8 +1852,12 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     cudaStream_t cs = (cudaStream_t)stream;
 
     cudaError_t e = cudaMemsetAsync(status_dev, 0, sizeof(int32_t), cs);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(sc->n_bits, n_bits_host, sizeof(int32_t) * (size_t)num_ctx, cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess) {
+        std::lock_guard<std::mutex> lock(g_noalloc_mu);
+        memcpy(g_noalloc_nbits, n_bits_host, sizeof(int32_t) * (size_t)num_ctx);
+        e = cudaMemcpyAsync(sc->n_bits, g_noalloc_nbits, sizeof(int32_t) * (size_t)num_ctx, cudaMemcpyHostToDevice,
+                            cs);
+    }
     if (e != cudaSuccess) return f2_cuda_status(e);
     noalloc_desc_kernel<<<1, 1024, 0, cs>>>(sc->n_bits, num_ctx, raw ? 1u : 0u, sc->desc);
 

@@ -50,6 +50,7 @@ __global__ void __launch_bounds__(256) merge_gather_kernel(StoreDev s, const int
 extern "C" int f2_merge_bases(const f2_store* src, int32_t num_groups, const int32_t* group_of,
                               const uint32_t* out_mask, f2_store** out, uint8_t* mask_ok, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_merge_bases");
     if (!out) return F2_ERR_INVALID_ARG;
     *out = nullptr;
     if (!src || num_groups < 0 || (src->num_ctx > 0 && !group_of)) return F2_ERR_INVALID_ARG;
@@ -102,7 +103,7 @@ extern "C" int f2_merge_bases(const f2_store* src, int32_t num_groups, const int
     uint32_t* d_x = nullptr;
     uint4* d_y = nullptr;
     auto am = [&](void** p, size_t bytes) {
-        if (e == cudaSuccess) e = cudaMallocAsync(p, bytes ? bytes : 16, cs);
+        if (e == cudaSuccess) e = f2_dev_alloc(src, p, bytes ? bytes : 16, cs, true);
     };
     am((void**)&d_row_off, sizeof(int64_t) * (size_t)(num_groups + 1));
     am((void**)&d_x_off, sizeof(int64_t) * x_off.size());

@@ -26,6 +26,7 @@ __global__ void __launch_bounds__(256) lop3_peak_kernel(uint32_t* out, int iters
 extern "C" int f2_peak_lop3(uint32_t* out_dev, int32_t blocks, int32_t iters, int64_t* lop3_per_launch,
                             f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_peak_lop3");
     if (!out_dev || blocks < 1 || iters < 1) return F2_ERR_INVALID_ARG;
     lop3_peak_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(out_dev, iters, 0x2545F491u);
     if (lop3_per_launch) *lop3_per_launch = (int64_t)blocks * 256 * (int64_t)iters * 8;

@@ -17,6 +17,19 @@ int f2_cuda_status(cudaError_t e)
 
 static inline bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
+cudaError_t f2_dev_alloc(const f2_store* st, void** p, size_t bytes, cudaStream_t cs, bool stream_ordered)
+{
+    if (st->fail_alloc_in >= 0) {
+        if (st->fail_alloc_in == 0) {  // the hooked allocation: fail once, then the hook is off
+            st->fail_alloc_in = -1;
+            *p = nullptr;
+            return cudaErrorMemoryAllocation;
+        }
+        --st->fail_alloc_in;
+    }
+    return stream_ordered ? cudaMallocAsync(p, bytes, cs) : cudaMalloc(p, bytes);
+}
+
 int f2_ensure_aux(const f2_store* st)
 {
     if (st->aux) return F2_OK;
@@ -87,6 +100,7 @@ static cudaError_t zero_state(f2_store* s, cudaStream_t st)
 extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
                          f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_create");
     if (!out) return F2_ERR_INVALID_ARG;
     *out = nullptr;
     if (num_ctx < 0 || (num_ctx > 0 && !n_bits_host) || (flags & ~F2_FLAG_RAW_FEATURES))
@@ -104,6 +118,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->enc_table_min = f2_encode_table_min_default();
     s->enc_chunk_shift = f2_encode_chunk_shift_default();
     s->enc_chunk_min = f2_encode_chunk_min_default();
+    s->fail_alloc_in = -1;
     s->host_chunk_bytes = DEFAULT_HOST_CHUNK_BYTES;
     if (cudaGetDevice(&s->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess) {
@@ -179,6 +194,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
 
 extern "C" void f2_destroy(f2_store* store)
 {
+    F2_NVTX_RANGE("f2_destroy");
     if (!store) return;
     cudaDeviceSynchronize();
     free_store(store);
@@ -186,6 +202,7 @@ extern "C" void f2_destroy(f2_store* store)
 
 extern "C" int f2_reset(f2_store* s, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_reset");
     if (!s) return F2_ERR_INVALID_ARG;
     return f2_cuda_status(zero_state(s, (cudaStream_t)stream));
 }
@@ -215,6 +232,7 @@ extern "C" int f2_get_basis(const f2_store* s, int32_t* rank, uint32_t* pivot_ma
                             uint32_t* basis_z, uint8_t* contra, int64_t* first_contra, uint64_t* n_contra,
                             int64_t* rows_seen, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_get_basis");
     if (!s) return F2_ERR_INVALID_ARG;
     cudaStream_t st = (cudaStream_t)stream;
     const size_t C = (size_t)s->num_ctx;
@@ -254,6 +272,7 @@ __global__ void __launch_bounds__(256) solve_kernel(StoreDev s, uint4* __restric
 
 extern "C" int f2_solve_affine(const f2_store* s, uint32_t* W, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_solve_affine");
     if (!s || (!W && s->slots)) return F2_ERR_INVALID_ARG;
     if (!aligned(W, 16)) return F2_ERR_ALIGN;
     if (s->num_ctx == 0) return F2_OK;
@@ -267,6 +286,7 @@ extern "C" int f2_solve_affine(const f2_store* s, uint32_t* W, f2_stream_t strea
 
 extern "C" int f2_device_status(f2_store* s, int* status, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_device_status");
     if (!s || !status) return F2_ERR_INVALID_ARG;
     cudaStream_t st = (cudaStream_t)stream;
     int v = 0;
@@ -302,6 +322,7 @@ size_t ckpt_size(const f2_store* s)
 
 extern "C" int f2_store_export(const f2_store* s, void* host_buf, size_t* size, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_store_export");
     if (!s || !size) return F2_ERR_INVALID_ARG;
     const size_t need = ckpt_size(s);
     if (!host_buf) {
@@ -345,6 +366,7 @@ extern "C" int f2_store_export(const f2_store* s, void* host_buf, size_t* size, 
 
 extern "C" int f2_store_import(f2_store* s, const void* host_buf, size_t size, f2_stream_t stream)
 {
+    F2_NVTX_RANGE("f2_store_import");
     if (!s || !host_buf) return F2_ERR_INVALID_ARG;
     const size_t need = ckpt_size(s);
     if (size < need) return F2_ERR_INVALID_ARG;
@@ -409,6 +431,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_ENCODE_CHUNK_MIN:
         if (value < 1) return F2_ERR_INVALID_ARG;
         s->enc_chunk_min = value;
+        return F2_OK;
+    case F2_OPT_FAIL_ALLOC:
+        if (value < -1) return F2_ERR_INVALID_ARG;
+        s->fail_alloc_in = value;
         return F2_OK;
     case F2_OPT_HOST_CHUNK_BYTES:
         if (value < (int64_t(1) << 16)) return F2_ERR_INVALID_ARG;
