@@ -789,6 +789,69 @@ def cpu_baseline(wl, seconds: float) -> dict:
                               "sample": f"{len(ctx1)} contexts ({rows1} rows), {t1:.1f} s"}}
 
 
+def _phase_summary(T, wl, b, e, smcol, ctx_ids):
+    has = T[:, e] > 0
+    if not has.any():
+        return None
+    beg, end, sm = T[has, b].astype(np.int64), T[has, e].astype(np.int64), T[has, smcol].astype(np.int64)
+    ids = ctx_ids[has]
+    t0 = int(beg.min())
+    span = int(end.max()) - t0
+    last = np.array([end[sm == k].max() - t0 for k in np.unique(sm)])
+    dur = end - beg
+    top = np.argsort(-dur)[:8]
+    return {
+        "contexts": int(has.sum()), "span_us": span / 1e3, "sms": int(len(last)),
+        "sm_finish_us": {"min": float(last.min()) / 1e3, "median": float(np.median(last)) / 1e3,
+                         "p90": float(np.percentile(last, 90)) / 1e3, "max": float(last.max()) / 1e3},
+        "tail_past_median_sm_frac": float((span - np.median(last)) / span),
+        "longest": [{"ctx": int(ids[k]), "rows": int(wl.rows[ids[k]]), "n": int(wl.n_bits[ids[k]]),
+                     "us": float(dur[k]) / 1e3, "start_us": float(beg[k] - t0) / 1e3,
+                     "end_us": float(end[k] - t0) / 1e3} for k in top],
+        "context_us_total": float(dur.sum()) / 1e3,
+    }
+
+
+def run_timing(args):
+    """Diagnostic (not the bench line): per-context timestamps of one learn
+    call (F2_OPT_TIMING) summarised per pass: how long the last context runs
+    past the median SM's last context, and the longest contexts."""
+    import torch
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2608_20532_gb300 import binding
+
+    dev = torch.device("cuda", 0)
+    wl = workload_for(args.config, 0, num_ctx=args.ctx)
+    t = lambda a: binding.to_device(a, dev)
+    x_t, y_t = t(wl.x), t(wl.y)
+    batches = [(t(ro), t(xo)) for ro, xo in wl.batches]
+    store = binding.Store(wl.n_bits, device=dev)
+    store.set_option(binding.F2_OPT_TIMING, 1)
+    for _ in range(args.warmup):
+        store.reset()
+        for ro, xo in batches:
+            store.learn(ro, x_t, xo, y_t)
+    torch.cuda.synchronize()
+    store.reset()
+    for ro, xo in batches[:-1]:
+        store.learn(ro, x_t, xo, y_t)
+    ro, xo = batches[-1]
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    store.learn(ro, x_t, xo, y_t)
+    ev[1].record()
+    torch.cuda.synchronize()
+    T = store.learn_timing()
+    ids = np.arange(wl.num_ctx)
+    out = {"config": describe(args.config, wl), "learn_call_ms": ev[0].elapsed_time(ev[1]),
+           "dedup": _phase_summary(T, wl, 0, 1, 4, ids), "elimination": _phase_summary(T, wl, 2, 3, 5, ids)}
+    if out["dedup"] and out["elimination"]:
+        out["dedup_end_to_elim_start_us"] = (int(T[T[:, 2] > 0, 2].min()) - int(T[T[:, 1] > 0, 1].max())) / 1e3
+    print(json.dumps(out), flush=True)
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -835,11 +898,15 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-probe", action="store_true")
+    ap.add_argument("--timing", action="store_true",
+                    help="diagnostic: per-context timestamps of one learn call, summarised (not the bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.timing:
+        run_timing(args)
     else:
         run_ours(args)
 

@@ -297,11 +297,26 @@ enum f2_option {
                                     default 20, in [11, 25]; raised so a pass has at most 64 chunks */
     F2_OPT_ENCODE_CHUNK_MIN = 8, /* fewest queries of one context (in a pass) for which its queries are
                                     laid out chunk by chunk (the others keep one run); default 1024 */
-    F2_OPT_FAIL_ALLOC = 9        /* test hook: the device allocation made after `value` more successful
+    F2_OPT_FAIL_ALLOC = 9,       /* test hook: the device allocation made after `value` more successful
                                     ones by calls on this store fails as if out of memory (the call
                                     returns F2_ERR_OOM; the store stays usable); -1 (default) = off */
+    F2_OPT_TIMING = 10,          /* 1: f2_learn_batched records per-context timestamps (f2_learn_timing);
+                                    0 (default): off */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
+
+/*
+ * Per-context timestamps of the last f2_learn_batched call on a store with
+ * F2_OPT_TIMING = 1 (a diagnostic with no counterpart in the paper: it shows
+ * how the contexts' work spreads over the SMs and how long the last context
+ * runs past the others).  out_host: host uint64[6*num_ctx]; for context c,
+ * words 6c..6c+3 are the device's %globaltimer (ns) at the start and end of
+ * the context's duplicate pass and of its elimination, words 6c+4 and 6c+5
+ * the ids of the SMs that ran them; zero where the context had no such work
+ * in that call.  Synchronizes `stream`.  Errors: F2_ERR_INVALID_ARG (NULL
+ * pointers, or no learn call with timing on), F2_ERR_CUDA.
+ */
+int f2_learn_timing(const f2_store* store, uint64_t* out_host, f2_stream_t stream);
 
 /*
  * Allocation-free learning (the paper has no counterpart; this is a

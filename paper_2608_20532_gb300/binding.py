@@ -37,13 +37,14 @@ F2_OPT_HOST_CHUNK_BYTES = 6
 F2_OPT_ENCODE_CHUNK_SHIFT = 7
 F2_OPT_ENCODE_CHUNK_MIN = 8
 F2_OPT_FAIL_ALLOC = 9
+F2_OPT_TIMING = 10
 
 # every entry point of include/f2gpu.h
 EXPORTS = (
     "f2_status_string", "f2_create", "f2_destroy", "f2_reset", "f2_layout", "f2_sizes",
     "f2_learn_batched", "f2_get_basis", "f2_solve_affine", "f2_encode_batched", "f2_device_status",
     "f2_store_export", "f2_store_import", "f2_set_option", "f2_peak_lop3", "f2_learn_batched_noalloc",
-    "f2_encode_epilogue", "f2_merge_bases", "f2_learn_host", "f2_encode_host",
+    "f2_encode_epilogue", "f2_merge_bases", "f2_learn_host", "f2_encode_host", "f2_learn_timing",
 )
 
 _lib = None
@@ -91,6 +92,7 @@ def load_library(path: Optional[str] = None):
         "f2_set_option": ([P, ctypes.c_int, i64], ctypes.c_int),
         "f2_peak_lop3": ([P, i32, i32, ctypes.POINTER(i64), P], ctypes.c_int),
         "f2_learn_batched_noalloc": ([i32, P, u32] + [P] * 9 + [P, P, P, P, i64, i64, P], ctypes.c_int),
+        "f2_learn_timing": ([P, P, P], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -296,6 +298,13 @@ class Store:
             if g[c] >= 0:
                 d[g[c]] = self.n_bits[c] + (0 if self.raw else 1)
         return Store(d, raw=True, device=self.device, _handle=h), ok[:int(num_groups)]
+
+    def learn_timing(self, stream=None) -> np.ndarray:
+        """Per-context timestamps of the last learn call (F2_OPT_TIMING on):
+        uint64[num_ctx, 6] = dedup start/end, elimination start/end (ns), their SM ids."""
+        out = np.zeros((self.num_ctx, 6), np.uint64)
+        _check(self._lib.f2_learn_timing(self._h, out.ctypes.data, _stream(stream)), "f2_learn_timing")
+        return out
 
     def device_status(self, stream=None) -> int:
         v = ctypes.c_int(0)

@@ -289,6 +289,9 @@ struct f2_store {
     // test hook (F2_OPT_FAIL_ALLOC): device allocations left before one is
     // made to fail; -1 = off
     mutable int64_t fail_alloc_in;
+    // diagnostics (F2_OPT_TIMING): per-context timestamps of the last learn call
+    int timing_on;
+    unsigned long long* timing;
     // host-input entry points (f2_learn_host, f2_encode_host)
     f2::HostIO* hio;
     int64_t host_chunk_bytes;               // bytes of rows (or queries) per copied chunk

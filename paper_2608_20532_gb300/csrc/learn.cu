@@ -62,6 +62,7 @@ struct LearnArgs {
     int* late_count;
     int32_t* late_list;
     int32_t* late_start;
+    unsigned long long* timing;  // per-context timestamps (F2_OPT_TIMING), NULL = off
 };
 
 struct DedupArgs {
@@ -74,7 +75,26 @@ struct DedupArgs {
     int32_t* rep_count;
     const int32_t* queue;
     int* counters;
+    unsigned long long* timing;  // per-context timestamps (F2_OPT_TIMING), NULL = off
 };
+
+// Per-context timestamps of a learn call (diagnostics, F2_OPT_TIMING):
+// TIME_WORDS words per context -- %globaltimer at the start and end of its
+// duplicate pass and of its elimination, then the SM ids that ran them.
+constexpr int TIME_WORDS = 6;
+__device__ __forceinline__ unsigned smid()
+{
+    unsigned r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void time_mark(unsigned long long* timing, int c, int slot)
+{
+    if (timing) {
+        timing[(size_t)TIME_WORDS * c + slot] = global_ns();
+        timing[(size_t)TIME_WORDS * c + 4 + (slot >> 1)] = smid();
+    }
+}
 
 // Shared-memory control area of an elimination group (32-bit words).
 constexpr int CTL_P = 0;       // pivot mask, 48 words
@@ -502,6 +522,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
             const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
             int E = pow2_at_least(2 * T);
             if (E > DD_CTA_E) E = DD_CTA_E;
+            if (threadIdx.x == 0) time_mark(a.timing, c, 0);
 #define F2_DD_CTA(W) dedup_ctx<DD_WARPS, W>(s, a, c, smem, E, wcnt)
             if constexpr (WX) {
                 F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_CTA)
@@ -509,6 +530,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
                 F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_CTA)
             }
 #undef F2_DD_CTA
+            if (threadIdx.x == 0) time_mark(a.timing, c, 1);
         }
     }
     {
@@ -526,6 +548,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
             const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
             int E = pow2_at_least(2 * T);
             if (E > DD_QUAD_E) E = DD_QUAD_E;
+            if ((warp & 3) == 0 && lane == 0) time_mark(a.timing, c, 0);
 #define F2_DD_QUAD(W) dedup_ctx<4, W>(s, a, c, region, E, wcnt + q * 4 * DD_K)
             if constexpr (WX) {
                 F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_QUAD)
@@ -533,6 +556,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
                 F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_QUAD)
             }
 #undef F2_DD_QUAD
+            if ((warp & 3) == 0 && lane == 0) time_mark(a.timing, c, 1);
         }
     }
     {
@@ -547,6 +571,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
             const int c = a.queue[b + item];
             const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
             const int E = pow2_at_least(2 * T);
+            if (lane == 0) time_mark(a.timing, c, 0);
 #define F2_DD_WARP(W) dedup_ctx<1, W>(s, a, c, region, E, nullptr)
             if constexpr (WX) {
                 F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_WARP)
@@ -554,6 +579,7 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
                 F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_WARP)
             }
 #undef F2_DD_WARP
+            if (lane == 0) time_mark(a.timing, c, 1);
         }
     }
 }
@@ -957,6 +983,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
         if (item >= n_cta) break;
         const int c = a.queue[b_cta + item];
         const int wd = s.desc[c].wd;
+        if (threadIdx.x == 0) time_mark(a.timing, c, 2);
 #define F2_CALL_CTA(W) elim_ctx<W, true>(s, a, c, smem)
         if (SMALL) {
             F2_SMALL_SWITCH(wd, F2_CALL_CTA)
@@ -964,6 +991,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
             F2_BIG_SWITCH(wd, F2_CALL_CTA)
         }
 #undef F2_CALL_CTA
+        if (threadIdx.x == 0) time_mark(a.timing, c, 3);
     }
     const int n_w = a.counters[CNT_COUNT + C_WARP];
     const int b_w = a.counters[CNT_BEGIN + C_WARP];
@@ -975,6 +1003,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
         if (item >= n_w) break;
         const int c = a.queue[b_w + item];
         const int wd = s.desc[c].wd;
+        if (lane == 0) time_mark(a.timing, c, 2);
 #define F2_CALL_WARP(W) elim_ctx<W, false>(s, a, c, region)
         if (SMALL) {
             F2_SMALL_SWITCH(wd, F2_CALL_WARP)
@@ -982,6 +1011,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
             F2_BIG_SWITCH(wd, F2_CALL_WARP)
         }
 #undef F2_CALL_WARP
+        if (lane == 0) time_mark(a.timing, c, 3);
     }
 }
 
@@ -1002,7 +1032,10 @@ __global__ void __launch_bounds__(WIDE_WARPS * 32, WDT <= WIDE_M_WD ? 2 : 1) eli
         __syncthreads();
         const int item = s_item;
         if (item >= n) break;
-        elim_ctx<WDT, true>(s, a, a.queue[b + item], smem);
+        const int c = a.queue[b + item];
+        if (threadIdx.x == 0) time_mark(a.timing, c, 2);
+        elim_ctx<WDT, true>(s, a, c, smem);
+        if (threadIdx.x == 0) time_mark(a.timing, c, 3);
     }
 }
 
@@ -1583,6 +1616,12 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (e != cudaSuccess) return F2_ERR_OOM;
         st->rep_capacity = total_rows;
     }
+    if (st->timing_on) {  // diagnostics: per-context timestamps of this call
+        const size_t bytes = sizeof(unsigned long long) * TIME_WORDS * (size_t)(st->num_ctx > 0 ? st->num_ctx : 1);
+        if (!st->timing && f2_dev_alloc(st, (void**)&st->timing, bytes, cs, true) != cudaSuccess) return F2_ERR_OOM;
+        e = cudaMemsetAsync(st->timing, 0, bytes, cs);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
     const StoreDev sd = st->dev();
     {
         const int rc = f2_ensure_aux(st);
@@ -1616,6 +1655,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         da.rep_count = st->rep_count;
         da.queue = st->queue;
         da.counters = st->counters;
+        da.timing = st->timing_on ? st->timing : nullptr;
         // the two instances hold disjoint contexts: side by side when both run
         const bool wide_rows = st->max_xw > DD_XW;  // some context has feature rows of 10..16 words
         e = cudaFuncSetAttribute(dedup_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
@@ -1645,6 +1685,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     la.rep_count = dedup ? st->rep_count : nullptr;
     la.queue = st->queue;
     la.counters = st->counters;
+    la.timing = st->timing_on ? st->timing : nullptr;
     la.warp_region_words = (int)(st->warp_basis_bytes / 4);
     if (!st->widths_ready) {  // fixed by the widths: computed once per store
         st->widths = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
@@ -1654,6 +1695,17 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
                               wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk);
+}
+
+extern "C" int f2_learn_timing(const f2_store* st, uint64_t* out_host, f2_stream_t stream)
+{
+    if (!st || !out_host) return F2_ERR_INVALID_ARG;
+    if (!st->timing) return F2_ERR_INVALID_ARG;  // no learn call since F2_OPT_TIMING was set
+    cudaStream_t cs = (cudaStream_t)stream;
+    cudaError_t e = cudaMemcpyAsync(out_host, st->timing, sizeof(uint64_t) * TIME_WORDS * (size_t)st->num_ctx,
+                                    cudaMemcpyDeviceToHost, cs);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(cs);
+    return f2_cuda_status(e);
 }
 
 // ---------------------------------------------------------------------------
@@ -1884,6 +1936,7 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     la.rep_count = nullptr;
     la.queue = sc->queue;
     la.counters = sc->counters;
+    la.timing = nullptr;
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
     const Widths wv = width_summary(n_bits_host, num_ctx, raw);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,

@@ -72,7 +72,7 @@ static void free_store(f2_store* s)
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
                     s->full_ctr, s->full_cnt, s->full_first,
                     s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items, s->enc_hot, s->enc_tab_off,
-                    s->enc_pool};
+                    s->enc_pool, s->timing};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     delete s;
@@ -435,6 +435,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_FAIL_ALLOC:
         if (value < -1) return F2_ERR_INVALID_ARG;
         s->fail_alloc_in = value;
+        return F2_OK;
+    case F2_OPT_TIMING:
+        if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
+        s->timing_on = (int)value;
         return F2_OK;
     case F2_OPT_HOST_CHUNK_BYTES:
         if (value < (int64_t(1) << 16)) return F2_ERR_INVALID_ARG;
