@@ -302,6 +302,11 @@ enum f2_option {
                                     returns F2_ERR_OOM; the store stays usable); -1 (default) = off */
     F2_OPT_TIMING = 10,          /* 1: f2_learn_batched records per-context timestamps (f2_learn_timing);
                                     0 (default): off */
+    F2_OPT_ELIM_TABLES = 11,     /* 1 (default): in contexts owned by a whole CTA, step (1) against a round's
+                                    snapshot uses a 4-bit lookup table of the basis where it fits and
+                                    pays; 0: always walk the pivots */
+    F2_OPT_SMALL_BASIS_BYTES = 12, /* shared memory (bytes) of one warp-owned context of width d <= 96;
+                                    default 4096, in [4096, 24576] */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -268,37 +268,13 @@ __global__ void __launch_bounds__(ENC_TILE_THREADS) enc_count_kernel(int32_t Q, 
 }
 
 // ---------------------------------------------------------------------------
-// Lookup tables (a Four-Russians table over 4-bit groups of coordinates).
-// The reduction of q against the reduced basis XORs, for every set
-// coordinate j of q, the vector E_j:
-//   j a pivot:     word part z_j, residual part r_j restricted to the
-//                  non-pivot coordinates (r_j has no other pivot bit);
-//   j not a pivot: word part 0, residual part the unit vector of j.
-// Residuals live on the m = d - rank non-pivot coordinates only, so they are
-// stored compressed (the t-th non-pivot coordinate in increasing order is
-// bit t).  E is linear in q, so for each group p of four coordinates the
-// table holds all 16 XOR combinations of E_{4p..4p+3}; a query then costs
-// exactly ceil(d/4) lookups and is in the span iff its compressed residual is
-// zero (Sec. 2.3: the word is T(q) = XOR of the z_k used; the query is
-// rejected otherwise).
-//
-// Layout of a table with np groups and rw residual words (word offsets):
-// low z half uint2[np*16] at 0, high z half at 32*np, residual word u
-// uint32[np*16] at 64*np + 16*np*u; entry e = 16*p + v.  With eight-byte and
-// four-byte planes the lookups of a warp at one position are free of bank
-// conflicts (the 16 values of v fall in distinct banks).  A table is
-// 16*np*(4 + rw) words, a multiple of 64 bytes.
+// Lookup tables of the basis (layout and meaning in f2_internal.cuh), built
+// once per pass for the contexts with many queries.
 // ---------------------------------------------------------------------------
-constexpr int TAB_WD = NARROW_WD;             // widest context with a table (d <= 288)
-constexpr int TAB_RW = 4;                     // compressed residual words (m <= 128)
+constexpr int TAB_WD = TABLE_MAX_WD;          // widest context with a table (d <= 288)
+constexpr int TAB_RW = TABLE_MAX_RW;          // compressed residual words (m <= 128)
 constexpr int TAB_WORDS = 6144;               // largest table (24 KB): one of two table buffers
 constexpr int DEFAULT_TABLE_MIN = 32;
-
-__host__ __device__ __forceinline__ int table_words(int d, int rank)
-{
-    const int np = (d + 3) >> 2, rw = (d - rank + 31) >> 5;
-    return 16 * np * (4 + rw);
-}
 
 // E_j of context cd: word part z, compressed residual er.  The pivot words,
 // z_j and r_j are loaded together (slots of non-pivots hold zeros), so an
@@ -731,42 +707,11 @@ __device__ __forceinline__ void load_x(const uint32_t* __restrict__ xq, int xw, 
 template <int RW, int WD>
 __device__ __forceinline__ bool table_query(const uint32_t* tab, int np, uint32_t (&q)[WD], uint4& acc)
 {
-    // one feature word (eight positions) per trip; q is consumed
-    const uint2* Zl = reinterpret_cast<const uint2*>(tab);
-    const uint2* Zh = Zl + np * 16;
-    const uint32_t* R = tab + 64 * np;
-    const int rstride = 16 * np;
-    uint32_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
     uint32_t r[RW > 0 ? RW : 1];
-#pragma unroll
-    for (int u = 0; u < (RW > 0 ? RW : 1); ++u) r[u] = 0;
-#pragma unroll 1
-    for (int left = np; left > 0; left -= 8) {
-        const uint32_t word = q[0];
-#pragma unroll
-        for (int v = 0; v < WD - 1; ++v) q[v] = q[v + 1];
-#pragma unroll
-        for (int h = 0; h < 8; ++h) {
-            if (h < left) {
-                const int e = h * 16 + (int)((word >> (4 * h)) & 15u);
-                const uint2 lo = Zl[e];
-                const uint2 hi = Zh[e];
-                a0 ^= lo.x;
-                a1 ^= lo.y;
-                a2 ^= hi.x;
-                a3 ^= hi.y;
-#pragma unroll
-                for (int u = 0; u < RW; ++u) r[u] ^= R[u * rstride + e];
-            }
-        }
-        Zl += 128;
-        Zh += 128;
-        R += 128;
-    }
+    table_reduce<RW, WD>(tab, np, q, acc, r);
     uint32_t res = 0;
 #pragma unroll
     for (int u = 0; u < RW; ++u) res |= r[u];
-    acc = make_uint4(a0, a1, a2, a3);
     return res == 0;
 }
 

@@ -31,6 +31,7 @@ constexpr int LEARN_WARPS = 8;       // warps per CTA of the narrow learn kernel
 constexpr int WIDE_WARPS = 8;        // warps per CTA of the wide learn kernel
 constexpr int PLAN_BUCKETS = 48;     // log2(work) buckets for longest-first ordering
 constexpr int DEFAULT_WARP_REGION_BYTES = 12288;  // shared memory of one warp-owned context
+constexpr int DEFAULT_SMALL_REGION_BYTES = 4096;  // the same in the small-width kernel (d <= 96)
 constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA
 constexpr long long DEFAULT_WARP_WORK = 131072;   // largest rows x d handled by one warp
 
@@ -104,6 +105,76 @@ struct StoreDev {
 // Shared-memory row stride (32-bit words) of a basis slot: the 128-bit z
 // first, then the wd feature words, padded to 16 bytes.
 __host__ __device__ constexpr int row_stride(int wd) { return 4 * ((4 + wd + 3) / 4); }
+
+// ---------------------------------------------------------------------------
+// Lookup tables of a reduced basis (a Four-Russians table over 4-bit groups
+// of coordinates), used by the encoder and by the elimination.  Reducing q
+// against the reduced basis XORs, for every set coordinate j of q, the vector
+// E_j:
+//   j a pivot:     word part z_j, residual part r_j restricted to the
+//                  non-pivot coordinates (r_j has no other pivot bit);
+//   j not a pivot: word part 0, residual part the unit vector of j.
+// Residuals live on the m = d - rank non-pivot coordinates only, so they are
+// stored compressed (the t-th non-pivot coordinate in increasing order is
+// bit t).  E is linear in q, so for each group p of four coordinates the
+// table holds all 16 XOR combinations of E_{4p..4p+3}; a reduction then
+// costs exactly ceil(d/4) lookups, and q lies in the span iff its compressed
+// residual is zero (Sec. 2.3; Sec. 2.2 step (1)).
+//
+// Layout of a table with np = ceil(d/4) groups and rw = ceil(m/32) residual
+// words (word offsets): low z half uint2[np*16] at 0, high z half at 32*np,
+// residual word u uint32[np*16] at 64*np + 16*np*u; entry e = 16*p + v.  With
+// eight-byte and four-byte planes the lookups of a warp at one position are
+// free of bank conflicts (the 16 values of v fall in distinct banks).  A
+// table is 16*np*(4 + rw) words, a multiple of 64 bytes.
+// ---------------------------------------------------------------------------
+constexpr int TABLE_MAX_WD = NARROW_WD;  // widest row with a table (d <= 288)
+constexpr int TABLE_MAX_RW = 4;          // compressed residual words (m <= 128)
+
+__host__ __device__ __forceinline__ int table_words(int d, int rank)
+{
+    const int np = (d + 3) >> 2, rw = (d - rank + 31) >> 5;
+    return 16 * np * (4 + rw);
+}
+
+// acc = XOR of the word parts, r = compressed residual of q (consumed: its
+// words are shifted out, eight coordinate groups per word).
+template <int RW, int WD>
+__device__ __forceinline__ void table_reduce(const uint32_t* tab, int np, uint32_t (&q)[WD], uint4& acc,
+                                             uint32_t (&r)[RW > 0 ? RW : 1])
+{
+    const uint2* Zl = reinterpret_cast<const uint2*>(tab);
+    const uint2* Zh = Zl + np * 16;
+    const uint32_t* R = tab + 64 * np;
+    const int rstride = 16 * np;
+    uint32_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+#pragma unroll
+    for (int u = 0; u < (RW > 0 ? RW : 1); ++u) r[u] = 0;
+#pragma unroll 1
+    for (int left = np; left > 0; left -= 8) {
+        const uint32_t word = q[0];
+#pragma unroll
+        for (int v = 0; v < WD - 1; ++v) q[v] = q[v + 1];
+#pragma unroll
+        for (int h = 0; h < 8; ++h) {
+            if (h < left) {
+                const int e = h * 16 + (int)((word >> (4 * h)) & 15u);
+                const uint2 lo = Zl[e];
+                const uint2 hi = Zh[e];
+                a0 ^= lo.x;
+                a1 ^= lo.y;
+                a2 ^= hi.x;
+                a3 ^= hi.y;
+#pragma unroll
+                for (int u = 0; u < RW; ++u) r[u] ^= R[u * rstride + e];
+            }
+        }
+        Zl += 128;
+        Zh += 128;
+        R += 128;
+    }
+    acc = make_uint4(a0, a1, a2, a3);
+}
 
 __device__ __forceinline__ void record_status(int* status, int code)
 {
@@ -234,6 +305,8 @@ struct f2_store {
     int64_t warp_basis_bytes;
     int64_t warp_work;
     int dedup;              // run the duplicate pass before elimination
+    int elim_tables;        // snapshot reduction by lookup table where it pays
+    int64_t small_basis_bytes;  // shared memory of a warp-owned context, small-width kernel
     f2::Widths widths;      // width classes of the contexts (computed on first use)
     // second stream of the learn launches (kernels of independent width
     // classes run side by side), its fork and join events; created on first use

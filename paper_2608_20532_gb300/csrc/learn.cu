@@ -63,6 +63,9 @@ struct LearnArgs {
     int32_t* late_list;
     int32_t* late_start;
     unsigned long long* timing;  // per-context timestamps (F2_OPT_TIMING), NULL = off
+    int tables;                  // reduce against a lookup table of the snapshot where it pays
+    int small_region_words;      // shared memory of a warp-owned context of the small-width kernel
+    int cta_region_words;        // shared memory of a CTA-owned context (the launch's dynamic size)
 };
 
 struct DedupArgs {
@@ -803,10 +806,207 @@ __device__ __forceinline__ void commit_stats(const StoreDev& s, int c, long long
 
 // ------------------------------------------------------------------ pass 2
 
+// Set compressed residual bit tt (< 32 * TABLE_MAX_RW).
+__device__ __forceinline__ void set_rbit(uint32_t (&er)[TABLE_MAX_RW], int tt)
+{
+#pragma unroll
+    for (int u = 0; u < TABLE_MAX_RW; ++u)
+        if ((tt >> 5) == u) er[u] |= 1u << (tt & 31);
+}
+
+constexpr int FL_WORDS = 64;  // free-coordinate list of a table: 128 uint16 entries
+
+// The lookup table (layout in f2_internal.cuh) of the basis held in shared
+// memory: pivot rows S (row stride row_stride(WD)), pivot mask P, rank; FL
+// receives the non-pivot coordinates in increasing order (the meaning of the
+// compressed residual bits).  All nt threads of the group take part.
+template <int WD, bool CTA>
+__device__ void build_table_smem(const uint32_t* __restrict__ S, const uint32_t (&P)[WD], int d, int wd, int rank,
+                                 uint32_t* __restrict__ TB, uint16_t* __restrict__ FL, int t, int nt)
+{
+    constexpr int RS = row_stride(WD);
+    const int np = (d + 3) >> 2, rw = (d - rank + 31) >> 5;
+    uint32_t f[WD];  // non-pivot coordinates of each word
+    int pre[WD];     // non-pivot coordinates in the words before
+    {
+        int acc = 0;
+#pragma unroll
+        for (int w = 0; w < WD; ++w) {
+            const uint32_t valid = (w < wd) ? ((w == wd - 1 && (d & 31)) ? ((1u << (d & 31)) - 1u) : 0xffffffffu) : 0u;
+            f[w] = ~P[w] & valid;
+            pre[w] = acc;
+            acc += __popc(f[w]);
+        }
+    }
+    uint2* const Zl = reinterpret_cast<uint2*>(TB);
+    uint2* const Zh = Zl + 16 * np;
+    uint32_t* const R = TB + 64 * np;
+    for (int j = t; j < 4 * np; j += nt) {
+        uint4 z = make_uint4(0, 0, 0, 0);
+        uint32_t er[TABLE_MAX_RW] = {0, 0, 0, 0};
+        if (j < d) {
+            const int w = j >> 5, b = j & 31;
+            uint32_t fw = 0;
+            int pw = 0;
+#pragma unroll
+            for (int u = 0; u < WD; ++u)
+                if (u == w) {
+                    fw = f[u];
+                    pw = pre[u];
+                }
+            if ((fw >> b) & 1u) {  // a non-pivot coordinate: its unit vector
+                const int tt = pw + __popc(fw & ((1u << b) - 1u));
+                set_rbit(er, tt);
+                FL[tt] = (uint16_t)j;
+            } else {  // a pivot: z_j and r_j on the non-pivot coordinates
+                const uint32_t* row = S + j * RS;
+                z = *reinterpret_cast<const uint4*>(row);
+#pragma unroll
+                for (int u = 0; u < WD; ++u) {
+                    if (u <= w) {
+                        uint32_t bits = row[4 + u] & f[u];
+                        while (bits) {
+                            const int bb = __ffs(bits) - 1;
+                            bits &= bits - 1u;
+                            set_rbit(er, pre[u] + __popc(f[u] & ((1u << bb) - 1u)));
+                        }
+                    }
+                }
+            }
+        }
+        const int e = 16 * (j >> 2) + (1 << (j & 3));
+        Zl[e] = make_uint2(z.x, z.y);
+        Zh[e] = make_uint2(z.z, z.w);
+#pragma unroll
+        for (int u = 0; u < TABLE_MAX_RW; ++u)
+            if (u < rw) R[u * 16 * np + e] = er[u];
+        if ((j & 3) == 0) {
+            const int e0 = 16 * (j >> 2);
+            Zl[e0] = make_uint2(0, 0);
+            Zh[e0] = make_uint2(0, 0);
+#pragma unroll
+            for (int u = 0; u < TABLE_MAX_RW; ++u)
+                if (u < rw) R[u * 16 * np + e0] = 0u;
+        }
+    }
+    group_sync<CTA>();
+    // entries of two or more coordinates: XOR of their single entries
+    for (int k = t; k < 16 * np; k += nt) {
+        const int v = k & 15;
+        if (__popc(v) < 2) continue;
+        const int eb = k & ~15;
+        uint2 lo = make_uint2(0, 0), hi = make_uint2(0, 0);
+        uint32_t rr[TABLE_MAX_RW] = {0, 0, 0, 0};
+#pragma unroll
+        for (int bb = 0; bb < 4; ++bb) {
+            if ((v >> bb) & 1) {
+                const int es = eb + (1 << bb);
+                const uint2 l = Zl[es], h = Zh[es];
+                lo.x ^= l.x;
+                lo.y ^= l.y;
+                hi.x ^= h.x;
+                hi.y ^= h.y;
+#pragma unroll
+                for (int u = 0; u < TABLE_MAX_RW; ++u)
+                    if (u < rw) rr[u] ^= R[u * 16 * np + es];
+            }
+        }
+        Zl[k] = lo;
+        Zh[k] = hi;
+#pragma unroll
+        for (int u = 0; u < TABLE_MAX_RW; ++u)
+            if (u < rw) R[u * 16 * np + k] = rr[u];
+    }
+    group_sync<CTA>();
+}
+
+// The full residual (feature words, zero at the pivots) from its compressed
+// form: bit tt is the non-pivot coordinate FL[tt].
+template <int WD>
+__device__ __forceinline__ void decompress_residual(const uint32_t (&cr)[TABLE_MAX_RW], int rw,
+                                                    const uint16_t* __restrict__ FL, uint32_t (&xr)[WD])
+{
+#pragma unroll
+    for (int v = 0; v < WD; ++v) xr[v] = 0u;
+#pragma unroll
+    for (int u = 0; u < TABLE_MAX_RW; ++u) {
+        uint32_t bits = (u < rw) ? cr[u] : 0u;
+        while (bits) {
+            const int bb = __ffs(bits) - 1;
+            bits &= bits - 1u;
+            const int coord = FL[32 * u + bb];
+#pragma unroll
+            for (int v = 0; v < WD; ++v)
+                if ((coord >> 5) == v) xr[v] |= 1u << (coord & 31);
+        }
+    }
+}
+
+// Snapshot reduction by table: acc of the word parts into yr, the residual
+// (zero at the pivots) into xr; returns whether it is nonzero.
+template <int WD>
+__device__ __forceinline__ bool reduce_by_table(uint32_t (&xr)[WD], uint4& yr, const uint32_t* __restrict__ TB,
+                                                const uint16_t* __restrict__ FL, int np, int rw)
+{
+    uint32_t q[WD];
+#pragma unroll
+    for (int v = 0; v < WD; ++v) q[v] = xr[v];
+    uint4 acc;
+    uint32_t cr[TABLE_MAX_RW] = {0, 0, 0, 0};
+    switch (rw) {
+    case 0: {
+        uint32_t r0[1];
+        table_reduce<0, WD>(TB, np, q, acc, r0);
+        break;
+    }
+    case 1: {
+        uint32_t r1[1];
+        table_reduce<1, WD>(TB, np, q, acc, r1);
+        cr[0] = r1[0];
+        break;
+    }
+    case 2: {
+        uint32_t r2[2];
+        table_reduce<2, WD>(TB, np, q, acc, r2);
+        cr[0] = r2[0];
+        cr[1] = r2[1];
+        break;
+    }
+    case 3: {
+        uint32_t r3[3];
+        table_reduce<3, WD>(TB, np, q, acc, r3);
+        cr[0] = r3[0];
+        cr[1] = r3[1];
+        cr[2] = r3[2];
+        break;
+    }
+    default: {
+        uint32_t r4[4];
+        table_reduce<4, WD>(TB, np, q, acc, r4);
+        cr[0] = r4[0];
+        cr[1] = r4[1];
+        cr[2] = r4[2];
+        cr[3] = r4[3];
+        break;
+    }
+    }
+    yr.x ^= acc.x;
+    yr.y ^= acc.y;
+    yr.z ^= acc.z;
+    yr.w ^= acc.w;
+    const bool nz = (cr[0] | cr[1] | cr[2] | cr[3]) != 0u;
+    if (nz) decompress_residual<WD>(cr, rw, FL, xr);
+    else {
+#pragma unroll
+        for (int v = 0; v < WD; ++v) xr[v] = 0u;
+    }
+    return nz;
+}
+
 // One group (a warp, or the whole CTA) streams the representatives of
 // context c through its basis.
 template <int WD, bool CTA>
-__device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t* region)
+__device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t* region, int region_words)
 {
     const int G = CTA ? (int)(blockDim.x >> 5) : 1;
     const int lane = threadIdx.x & 31;
@@ -841,6 +1041,14 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
 #pragma unroll
     for (int v = 0; v < WD; ++v) P[v] = Ps[v];
     uint64_t mixed = mixed_words<WD>(P, cd.d, cd.wd);
+    // lookup table of the snapshot (rebuilt after a round that inserted):
+    // after the basis rows, the free-coordinate list at the region's end
+    constexpr int RS = row_stride(WD);
+    uint32_t* const TB = S + cd.d * RS;
+    uint16_t* const FL = reinterpret_cast<uint16_t*>(region + region_words - FL_WORDS);
+    const int tab_cap = region_words - FL_WORDS - CTL_WORDS - cd.d * RS;
+    const int np = (cd.d + 3) >> 2;
+    bool dirty = true;
     const long long seen = s.rows_seen[c];
     const int64_t r0 = a.row_off[c];
     const int64_t T = a.row_off[c + 1] - r0;
@@ -862,7 +1070,8 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     uint4 yn;
     load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
     int stop_at = -1;
-    for (int base = 0; base < R; base += nt) {
+    int parity = 0;
+    for (int base = 0; base < R; base += nt, parity ^= 1) {
         const bool valid = nvalid;
         const int i = ni;
         const uint32_t weight = 1u + nw;
@@ -874,12 +1083,37 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
         ni = nvalid ? (reps ? __ldg(reps + nk) : nk) : 0;
         nw = (nvalid && dups) ? (uint32_t)__ldg(dups + nk) : 0u;
         load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
-        reduce_snapshot<WD>(xr, yr, S, P, mixed);
+        // step (1) against the snapshot: by lookup table where the table fits
+        // and costs fewer instructions than walking the pivots (about d/4
+        // lookups a row against about rank/2 two-pivot steps), else by walk
+        int tmode = 0;  // 1 + residual words of the table, 0 = walk
+        // (CTA-owned contexts only: their many rounds after the basis stops
+        // growing repay the rebuilds; a warp-owned context has few rounds,
+        // most of them inserting, and keeps the small shared-memory region
+        // that lets more warps run)
+        if constexpr (CTA && WD <= TABLE_MAX_WD) {
+            if (a.tables) {
+                const int rk = *rank_s;
+                const int rw = (cd.d - rk + 31) >> 5;
+                if (rw <= TABLE_MAX_RW && table_words(cd.d, rk) <= tab_cap && 4 * rk >= 5 * np) {
+                    tmode = 1 + rw;
+                    if (dirty) {
+                        build_table_smem<WD, CTA>(S, P, cd.d, cd.wd, rk, TB, FL, t, nt);
+                        dirty = false;
+                    }
+                }
+            }
+        }
         uint32_t nz = 0;
+        if (tmode) {
+            nz = reduce_by_table<WD>(xr, yr, TB, FL, np, tmode - 1) ? 1u : 0u;
+        } else {
+            reduce_snapshot<WD>(xr, yr, S, P, mixed);
 #pragma unroll
-        for (int v = 0; v < WD; ++v) {
-            xr[v] &= ~P[v];
-            nz |= xr[v];
+            for (int v = 0; v < WD; ++v) {
+                xr[v] &= ~P[v];
+                nz |= xr[v];
+            }
         }
         bool contra_lane = false;
         if (valid && !nz && nonzero4(yr)) {
@@ -890,11 +1124,15 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
         const uint32_t cand = __ballot_sync(FULL, valid && nz != 0u);
         uint32_t wmask;
         if (CTA) {
-            if (lane == 0) wc[warp] = cand;
+            // two alternating ballot buffers: a round without candidates
+            // ends without a barrier, so the next round's ballots must not
+            // overwrite this round's before every warp has read them
+            uint32_t* const wcp = wc + 16 * parity;
+            if (lane == 0) wcp[warp] = cand;
             __syncthreads();
             wmask = 0;
             for (int ww = 0; ww < G; ++ww)
-                if (wc[ww]) wmask |= 1u << ww;
+                if (wcp[ww]) wmask |= 1u << ww;
         } else {
             wmask = cand ? 1u : 0u;
         }
@@ -921,6 +1159,7 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
                 for (int v = 0; v < WD; ++v) P[v] = Ps[v];
             }
             mixed = mixed_words<WD>(P, cd.d, cd.wd);
+            dirty = true;
             if (CTA) {
                 if (t < 48) NPR[t] = 0u;
             }
@@ -961,8 +1200,7 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
 // warp-owned ones.  SMALL: the contexts of at most SMALL_WD words, with
 // fixed 4 KB warp regions and a register budget for four CTAs per SM; else
 // the contexts of SMALL_WD + 1 .. NARROW_WD words.
-constexpr int SMALL_REGION_WORDS = 1024;
-static_assert(SMALL_REGION_WORDS >= 32 * SMALL_WD * row_stride(SMALL_WD) + CTL_WORDS,
+static_assert(DEFAULT_SMALL_REGION_BYTES / 4 >= 32 * SMALL_WD * row_stride(SMALL_WD) + CTL_WORDS + FL_WORDS,
               "a warp region holds the basis of any small-width context");
 
 template <bool SMALL>
@@ -984,7 +1222,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
         const int c = a.queue[b_cta + item];
         const int wd = s.desc[c].wd;
         if (threadIdx.x == 0) time_mark(a.timing, c, 2);
-#define F2_CALL_CTA(W) elim_ctx<W, true>(s, a, c, smem)
+#define F2_CALL_CTA(W) elim_ctx<W, true>(s, a, c, smem, a.cta_region_words)
         if (SMALL) {
             F2_SMALL_SWITCH(wd, F2_CALL_CTA)
         } else {
@@ -995,7 +1233,8 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
     }
     const int n_w = a.counters[CNT_COUNT + C_WARP];
     const int b_w = a.counters[CNT_BEGIN + C_WARP];
-    uint32_t* region = smem + warp * (SMALL ? SMALL_REGION_WORDS : a.warp_region_words);
+    const int region_words = SMALL ? a.small_region_words : a.warp_region_words;
+    uint32_t* region = smem + warp * region_words;
     for (;;) {
         int item = 0;
         if (lane == 0) item = atomicAdd(a.counters + CNT_HEAD + C_WARP, 1);
@@ -1004,7 +1243,7 @@ __global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_k
         const int c = a.queue[b_w + item];
         const int wd = s.desc[c].wd;
         if (lane == 0) time_mark(a.timing, c, 2);
-#define F2_CALL_WARP(W) elim_ctx<W, false>(s, a, c, region)
+#define F2_CALL_WARP(W) elim_ctx<W, false>(s, a, c, region, region_words)
         if (SMALL) {
             F2_SMALL_SWITCH(wd, F2_CALL_WARP)
         } else {
@@ -1034,7 +1273,7 @@ __global__ void __launch_bounds__(WIDE_WARPS * 32, WDT <= WIDE_M_WD ? 2 : 1) eli
         if (item >= n) break;
         const int c = a.queue[b + item];
         if (threadIdx.x == 0) time_mark(a.timing, c, 2);
-        elim_ctx<WDT, true>(s, a, c, smem);
+        elim_ctx<WDT, true>(s, a, c, smem, a.cta_region_words);
         if (threadIdx.x == 0) time_mark(a.timing, c, 3);
     }
 }
@@ -1487,7 +1726,9 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, LEARN_WARPS * 32, smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         if (per_sm < 1) per_sm = 1;
-        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, ks>>>(sd, lx);
+        LearnArgs lk = lx;
+        lk.cta_region_words = (int)(smem / 4);
+        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, ks>>>(sd, lk);
         return f2_cuda_status(cudaGetLastError());
     };
     // the three width classes hold disjoint contexts: with a second stream
@@ -1505,7 +1746,9 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         if (per_sm < 1) per_sm = 1;
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
-        kernel<<<num_sms * per_sm, WIDE_WARPS * 32, smem, ks>>>(sd, lx);
+        LearnArgs lk = lx;
+        lk.cta_region_words = (int)(smem / 4);
+        kernel<<<num_sms * per_sm, WIDE_WARPS * 32, smem, ks>>>(sd, lk);
         return f2_cuda_status(cudaGetLastError());
     };
     if (wv.has_wide) {
@@ -1523,7 +1766,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         if (rc != F2_OK) return rc;
     }
     if (wv.has_small) {
-        const size_t words = (size_t)LEARN_WARPS * SMALL_REGION_WORDS;
+        const size_t words = (size_t)LEARN_WARPS * (size_t)la.small_region_words;
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
         rc = narrow(elim_narrow_kernel<true>,
@@ -1687,6 +1930,9 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     la.counters = st->counters;
     la.timing = st->timing_on ? st->timing : nullptr;
     la.warp_region_words = (int)(st->warp_basis_bytes / 4);
+    la.tables = st->elim_tables;
+    la.small_region_words = (int)(st->small_basis_bytes / 4);
+    la.cta_region_words = 0;  // set per launch
     if (!st->widths_ready) {  // fixed by the widths: computed once per store
         st->widths = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
         st->widths_ready = true;
@@ -1937,6 +2183,9 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     la.queue = sc->queue;
     la.counters = sc->counters;
     la.timing = nullptr;
+    la.tables = 1;
+    la.small_region_words = DEFAULT_SMALL_REGION_BYTES / 4;
+    la.cta_region_words = 0;
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
     const Widths wv = width_summary(n_bits_host, num_ctx, raw);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,

@@ -115,6 +115,8 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->warp_basis_bytes = DEFAULT_WARP_REGION_BYTES;
     s->warp_work = DEFAULT_WARP_WORK;
     s->dedup = 1;
+    s->elim_tables = 1;
+    s->small_basis_bytes = DEFAULT_SMALL_REGION_BYTES;
     s->enc_table_min = f2_encode_table_min_default();
     s->enc_chunk_shift = f2_encode_chunk_shift_default();
     s->enc_chunk_min = f2_encode_chunk_min_default();
@@ -435,6 +437,14 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_FAIL_ALLOC:
         if (value < -1) return F2_ERR_INVALID_ARG;
         s->fail_alloc_in = value;
+        return F2_OK;
+    case F2_OPT_ELIM_TABLES:
+        if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
+        s->elim_tables = (int)value;
+        return F2_OK;
+    case F2_OPT_SMALL_BASIS_BYTES:
+        if (value < 4096 || value > 24576) return F2_ERR_INVALID_ARG;
+        s->small_basis_bytes = (value / 16) * 16;
         return F2_OK;
     case F2_OPT_TIMING:
         if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
