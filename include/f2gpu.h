@@ -282,9 +282,14 @@ int f2_store_import(f2_store* store, const void* host_buf, size_t size, f2_strea
 
 /* Scheduling knobs of f2_learn_batched (performance only, never results). */
 enum f2_option {
-    F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA */
+    F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA; unless
+                                this or F2_OPT_WARP_WORK is set, the call scales both to its own work
+                                (representatives / (20 SMs), within [1024, 4096]; with the duplicate
+                                pass off, rows / 20000) */
     F2_OPT_WARP_BASIS_BYTES = 2, /* shared memory (bytes) of one warp-owned context */
-    F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context */
+    F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context; default 131072,
+                                    scaled like F2_OPT_HEAVY_ROWS (sum of rows x d / (45 SMs), at least
+                                    32768) */
     F2_OPT_DEDUP = 4,            /* 1 (default): eliminate only the first occurrence of each distinct
                                     row and classify its repeats with it; 0: eliminate every row */
     F2_OPT_ENCODE_TABLE_MIN = 5, /* fewest queries of one context (in a pass of f2_encode_batched)

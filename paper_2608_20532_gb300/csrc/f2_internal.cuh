@@ -32,7 +32,12 @@ constexpr int WIDE_WARPS = 8;        // warps per CTA of the wide learn kernel
 constexpr int PLAN_BUCKETS = 48;     // log2(work) buckets for longest-first ordering
 constexpr int DEFAULT_WARP_REGION_BYTES = 12288;  // shared memory of one warp-owned context
 constexpr int DEFAULT_SMALL_REGION_BYTES = 4096;  // the same in the small-width kernel (d <= 96)
-constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA
+constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA (at most)
+constexpr int HEAVY_ROWS_MIN = 1024;              // ... and at least, when it scales with the batch:
+constexpr int HEAVY_ROWS_BATCH_DIV = 20000;       // batch rows / this (no duplicate pass), or
+constexpr int HEAVY_REPS_DIV = 20;                // representatives / (SMs x this) after the duplicate pass
+constexpr long long WARP_WORK_MIN = 32768;        // scaled warp work (rows x d) stays within
+constexpr int WARP_WORK_DIV = 45;                 // [this, the option]: sum(rows x d) / (SMs x this)
 constexpr long long DEFAULT_WARP_WORK = 131072;   // largest rows x d handled by one warp
 
 // Scheduling counters written by the plan kernel, read by the learn kernels.
@@ -40,7 +45,9 @@ enum Counter {
     CNT_HEAD = 0,   // + class: next queue item of each class
     CNT_BEGIN = 16, // + class: first queue slot of each class
     CNT_COUNT = 32, // + class: number of contexts of each class
-    CNT_WORDS = 48
+    CNT_WORK = 48,  // (uint64) sum over contexts of representatives x d, from the duplicate pass
+    CNT_REPS = 50,  // (uint64) sum of the representatives
+    CNT_WORDS = 52
 };
 // Work classes: elimination by a CTA / the wide kernel / a warp, dedup by a
 // CTA / a quad of warps / a warp, elimination of the small-width contexts
@@ -302,6 +309,8 @@ struct f2_store {
     int64_t basis_words;
     int64_t pivot_words;
     int64_t heavy_rows;
+    int heavy_rows_set;     // F2_OPT_HEAVY_ROWS given explicitly (else it scales with the batch)
+    int warp_work_set;      // F2_OPT_WARP_WORK given explicitly
     int64_t warp_basis_bytes;
     int64_t warp_work;
     int dedup;              // run the duplicate pass before elimination

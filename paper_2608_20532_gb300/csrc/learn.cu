@@ -489,7 +489,13 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
         const int slot = a.rep_dup[r0 + k];
         a.rep_dup[r0 + k] = (slot >= 0) ? D[slot] : 0;
     }
-    if (t == 0) a.rep_count[c] = nrep;
+    if (t == 0) {
+        a.rep_count[c] = nrep;
+        // the call's work, for the elimination plan's thresholds
+        atomicAdd(reinterpret_cast<unsigned long long*>(a.counters + CNT_WORK),
+                  (unsigned long long)nrep * (unsigned long long)cd.d);
+        atomicAdd(reinterpret_cast<unsigned long long*>(a.counters + CNT_REPS), (unsigned long long)nrep);
+    }
     dd_sync<G>();
 }
 
@@ -1304,6 +1310,8 @@ struct PlanArgs {
     int warp_region_words;
     int64_t heavy_rows;
     int64_t warp_work;
+    int scale;     // mode 1: scale heavy_rows / warp_work to the totals of the duplicate pass
+    int num_sms;
     int32_t* queue;
     int32_t* keybuf;
     int* hist;     // PLAN_KEYS counts (zeroed before plan_key_kernel), then cursors
@@ -1315,6 +1323,18 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
     __shared__ int hist[PLAN_KEYS];
     for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x) hist[i] = 0;
     __syncthreads();
+    // ownership thresholds, scaled to the call's work when the duplicate
+    // pass has measured it: a warp-owned context must not run (dependent
+    // round after round) much longer than the whole call
+    long long heavy_rows = p.heavy_rows, warp_work = p.warp_work;
+    if (p.mode == 1 && p.scale) {
+        const unsigned long long tw = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_WORK);
+        const unsigned long long tr = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_REPS);
+        const long long hr = (long long)(tr / ((unsigned long long)p.num_sms * HEAVY_REPS_DIV));
+        const long long ww = (long long)(tw / ((unsigned long long)p.num_sms * WARP_WORK_DIV));
+        heavy_rows = hr < HEAVY_ROWS_MIN ? HEAVY_ROWS_MIN : (hr > heavy_rows ? heavy_rows : hr);
+        warp_work = ww < WARP_WORK_MIN ? WARP_WORK_MIN : (ww > warp_work ? warp_work : ww);
+    }
     for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
         const CtxDesc cd = s.desc[c];
         int64_t R;
@@ -1349,8 +1369,8 @@ __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
                 if (cd.xw > DD_XW) cls += CLS_DDW_CTA - CLS_DD_CTA;  // the 10..16-word instance
                 work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
             } else {
-                const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= p.heavy_rows ||
-                                   R * cd.d > p.warp_work;
+                const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= heavy_rows ||
+                                   R * cd.d > warp_work;
                 if (s.rank[c] == cd.d) cls = CLS_FULL;
                 else if (cd.wd > NARROW_WD) cls = (cd.wd <= WIDE_M_WD) ? CLS_WIDE_M : CLS_WIDE;
                 else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
@@ -1689,7 +1709,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
-                       unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr)
+                       unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr, int scale = 0)
 {
     // full_ctr: chunks claimed [C], chunks done [C], late start [C], late list [C], late count
     const int C = sd.num_ctx;
@@ -1712,6 +1732,8 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     pa.warp_region_words = la.warp_region_words;
     pa.heavy_rows = heavy_rows;
     pa.warp_work = warp_work;
+    pa.scale = scale;
+    pa.num_sms = num_sms;
     pa.queue = queue;
     pa.keybuf = keybuf;
     pa.hist = hist;
@@ -1872,6 +1894,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     Fork fk{cs, st->aux, st->ev_fork, st->ev_join};
     if (dedup) {
+        e = cudaMemsetAsync(st->counters + CNT_WORK, 0, 4 * sizeof(int), cs);  // the work totals
+        if (e != cudaSuccess) return f2_cuda_status(e);
         PlanArgs pa;
         pa.row_off = row_off;
         pa.x_off = x_off;
@@ -1882,6 +1906,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         pa.warp_region_words = 0;
         pa.heavy_rows = 0;
         pa.warp_work = 0;
+        pa.scale = 0;
+        pa.num_sms = st->num_sms;
         pa.queue = st->queue;
         pa.keybuf = st->keybuf;
         pa.hist = st->plan_hist;
@@ -1938,9 +1964,20 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         st->widths_ready = true;
     }
     const Widths& wv = st->widths;
+    // Rows from which a context gets a whole CTA: unless set explicitly, it
+    // scales with the batch -- in a short call a warp-owned context of a few
+    // thousand rows, dependent round after round, would outlast everything
+    // else, while in a long one warps keep the SMs fuller
+    int64_t heavy = st->heavy_rows;
+    if (!st->heavy_rows_set && !dedup) {
+        heavy = total_rows / HEAVY_ROWS_BATCH_DIV;
+        if (heavy < HEAVY_ROWS_MIN) heavy = HEAVY_ROWS_MIN;
+        if (heavy > st->heavy_rows) heavy = st->heavy_rows;
+    }
+    const int scale = dedup && !st->heavy_rows_set && !st->warp_work_set;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
-                              st->heavy_rows, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms,
-                              wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk);
+                              heavy, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms, wv,
+                              st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale);
 }
 
 extern "C" int f2_learn_timing(const f2_store* st, uint64_t* out_host, f2_stream_t stream)

@@ -36,7 +36,12 @@ int f2_ensure_aux(const f2_store* st)
     int cur = -1;  // created on the store's device
     cudaError_t e = cudaGetDevice(&cur);
     if (e == cudaSuccess && cur != st->device) e = cudaSetDevice(st->device);
-    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
+    // the second stream carries the kernel of the heaviest width class (the
+    // wide or the 4..9-word elimination): at the highest priority its CTAs,
+    // and so its longest contexts, are dispatched first
+    int least = 0, greatest = 0;
+    if (e == cudaSuccess) e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
+    if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&st->aux, cudaStreamNonBlocking, greatest);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_fork, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_join, cudaEventDisableTiming);
     if (cur >= 0 && cur != st->device) cudaSetDevice(cur);
@@ -409,6 +414,7 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_HEAVY_ROWS:
         if (value < 1) return F2_ERR_INVALID_ARG;
         s->heavy_rows = value;
+        s->heavy_rows_set = 1;
         return F2_OK;
     case F2_OPT_WARP_BASIS_BYTES:
         if (value < 0 || value > 24576) return F2_ERR_INVALID_ARG;
@@ -417,6 +423,7 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_WARP_WORK:
         if (value < 0) return F2_ERR_INVALID_ARG;
         s->warp_work = value;
+        s->warp_work_set = 1;
         return F2_OK;
     case F2_OPT_DEDUP:
         if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;
