@@ -293,7 +293,7 @@ enum f2_option {
     F2_OPT_DEDUP = 4,            /* 1 (default): eliminate only the first occurrence of each distinct
                                     row and classify its repeats with it; 0: eliminate every row */
     F2_OPT_ENCODE_TABLE_MIN = 5, /* fewest queries of one context (in a pass of f2_encode_batched)
-                                    for which a lookup table of its basis is built; default 32, at
+                                    for which a lookup table of its basis is built; default 64, at
                                     least 1; a value above the pass size disables the tables */
     F2_OPT_HOST_CHUNK_BYTES = 6, /* bytes of rows (f2_learn_host) or of queries (f2_encode_host) per
                                     copied chunk; default 512 MiB, at least 64 KiB */
@@ -301,7 +301,7 @@ enum f2_option {
                                     written together (L2 locality of f2_encode_batched's output);
                                     default 20, in [11, 25]; raised so a pass has at most 64 chunks */
     F2_OPT_ENCODE_CHUNK_MIN = 8, /* fewest queries of one context (in a pass) for which its queries are
-                                    laid out chunk by chunk (the others keep one run); default 1024 */
+                                    laid out chunk by chunk (the others keep one run); default 512 */
     F2_OPT_FAIL_ALLOC = 9,       /* test hook: the device allocation made after `value` more successful
                                     ones by calls on this store fails as if out of memory (the call
                                     returns F2_ERR_OOM; the store stays usable); -1 (default) = off */

@@ -146,7 +146,7 @@ constexpr int32_t EMPTY_KEY = -1;
 constexpr int TBL_THREADS = 256;
 constexpr uint8_t HOT_TABLE = 1;    // the context's runs are encoded with its table
 constexpr uint8_t HOT_CHUNKED = 2;  // the context's queries are laid out chunk by chunk
-constexpr int64_t DEFAULT_CHUNK_MIN = 1024;
+constexpr int64_t DEFAULT_CHUNK_MIN = 512;
 constexpr int64_t POOL_MAX_WORDS = int64_t(1) << 28;  // table pool cap (1 GiB)
 static_assert(ENC_TILE <= (1 << ENC_MIN_SHIFT), "count tiles never straddle a chunk");
 
@@ -274,7 +274,7 @@ __global__ void __launch_bounds__(ENC_TILE_THREADS) enc_count_kernel(int32_t Q, 
 constexpr int TAB_WD = TABLE_MAX_WD;          // widest context with a table (d <= 288)
 constexpr int TAB_RW = TABLE_MAX_RW;          // compressed residual words (m <= 128)
 constexpr int TAB_WORDS = 6144;               // largest table (24 KB): one of two table buffers
-constexpr int DEFAULT_TABLE_MIN = 32;
+constexpr int DEFAULT_TABLE_MIN = 64;
 
 // E_j of context cd: word part z, compressed residual er.  The pivot words,
 // z_j and r_j are loaded together (slots of non-pivots hold zeros), so an

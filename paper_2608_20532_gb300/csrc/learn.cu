@@ -1467,7 +1467,6 @@ int launch_plan(const StoreDev& sd, const PlanArgs& pa, int num_sms, cudaStream_
 
 inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) == 0; }
 
-// Shared-memory need of the narrow elimination kernel for a set of widths.
 // ---------------------------------------------------------------------------
 // Full-rank contexts.  When rank = d at the start of a call the reduced basis
 // is the identity (every coordinate is a pivot and a reduced row has no other
