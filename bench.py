@@ -733,18 +733,22 @@ def run_ours(args):
 
 
 def launches_per_step(wl, has_q: bool) -> int:
-    """Kernels one step enqueues (the host logic of the library): per learn
-    call a plan (3 kernels) and dedup_kernel (a second instance when some
-    feature row has more than 9 words) for the duplicate pass, a plan,
+    """Kernels one step enqueues (the host logic of the library): the reset's
+    fill; per learn call the fill of its counters, a plan (one kernel for at
+    most 8,192 contexts, else three) and dedup_kernel (a second instance when
+    some feature row has more than 9 words) for the duplicate pass, a plan,
     the elimination kernel of each width class present (d <= 96, 96 < d <=
     288, 288 < d <= 544, wider) and the full-rank check; solve_kernel; per
-    2^25 queries the five encode kernels."""
+    2^25 queries the encode's fill and its seven kernels (count, table,
+    build, scan, scatter, runs, short)."""
     wd = (wl.n_bits.astype(np.int64) + 1 + 31) // 32
     xw = (wl.n_bits.astype(np.int64) + 31) // 32
-    learn = (3 + 1 + int((xw > 9).any()) + 3 + int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any())
-             + int(((wd > 9) & (wd <= 17)).any()) + int((wd > 17).any()) + 1)
-    enc = 5 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
-    return len(wl.batches) * learn + 1 + enc
+    plan = 1 if wl.num_ctx <= 8192 else 3
+    elim = (int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any()) + int(((wd > 9) & (wd <= 17)).any())
+            + int((wd > 17).any()))
+    learn = 1 + plan + 1 + int((xw > 9).any()) + plan + elim + 1
+    enc = 8 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
+    return 1 + len(wl.batches) * learn + 1 + enc
 
 
 def basis_bytes_touched(wl, store) -> int:

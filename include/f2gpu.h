@@ -312,6 +312,11 @@ enum f2_option {
                                     pays; 0: always walk the pivots */
     F2_OPT_SMALL_BASIS_BYTES = 12, /* shared memory (bytes) of one warp-owned context of width d <= 96;
                                     default 4096, in [4096, 24576] */
+    F2_OPT_DEDUP_SHARDS = 13,    /* most CTAs that the duplicate pass of one context is split over
+                                    (consecutive row ranges of at least 2048 rows: one per 1/(4 x SMs)
+                                    of the call's rows x (feature words + 4) the context holds, and
+                                    at least one per 16384 rows); default 4, in [1, 8]; 1 = never
+                                    split (and no 4-warp context promoted to a whole CTA) */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -40,6 +40,7 @@ F2_OPT_FAIL_ALLOC = 9
 F2_OPT_TIMING = 10
 F2_OPT_ELIM_TABLES = 11
 F2_OPT_SMALL_BASIS_BYTES = 12
+F2_OPT_DEDUP_SHARDS = 13
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

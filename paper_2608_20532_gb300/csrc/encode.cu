@@ -1293,11 +1293,15 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
         const int32_t Tn = (int32_t)((sn + SCAN_TILE - 1) / SCAN_TILE);
         const uint32_t* xq = x + q0 * x_stride_words;
         uint4* yq = reinterpret_cast<uint4*>(y_out) + q0;
-        e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * (size_t)(nch * B), cs);
-        if (e == cudaSuccess) e = cudaMemsetAsync(ticket, 0, 2 * sizeof(int32_t), cs);
-        if (e == cudaSuccess) e = cudaMemsetAsync(n_hot, 0, sizeof(int32_t), cs);
-        if (e == cudaSuccess) e = cudaMemsetAsync(pool_used, 0, sizeof(unsigned long long), cs);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        {  // the pass's counters, one launch
+            F2FillList zl;
+            zl.add(cnt, sizeof(int32_t) * (size_t)(nch * B));
+            zl.add(ticket, 2 * sizeof(int32_t));
+            zl.add(n_hot, sizeof(int32_t));
+            zl.add(pool_used, sizeof(unsigned long long));
+            e = f2_fill(zl, cs);
+            if (e != cudaSuccess) return f2_cuda_status(e);
+        }
         enc_count_kernel<<<(n + ENC_TILE - 1) / ENC_TILE, ENC_TILE_THREADS, 0, cs>>>(n, ctx_id + q0, st->num_ctx,
                                                                                    shift, (int32_t)B, cnt,
                                                                                    st->enc_off);

@@ -47,7 +47,8 @@ enum Counter {
     CNT_COUNT = 32, // + class: number of contexts of each class
     CNT_WORK = 48,  // (uint64) sum over contexts of representatives x d, from the duplicate pass
     CNT_REPS = 50,  // (uint64) sum of the representatives
-    CNT_WORDS = 52
+    CNT_SHARDS = 52,  // shard items beyond one per context claimed by the duplicate-pass plan
+    CNT_WORDS = 54
 };
 // Work classes: elimination by a CTA / the wide kernel / a warp, dedup by a
 // CTA / a quad of warps / a warp, elimination of the small-width contexts
@@ -316,6 +317,7 @@ struct f2_store {
     int dedup;              // run the duplicate pass before elimination
     int elim_tables;        // snapshot reduction by lookup table where it pays
     int64_t small_basis_bytes;  // shared memory of a warp-owned context, small-width kernel
+    int dd_shards;              // most CTAs one context's duplicate pass is split over
     f2::Widths widths;      // width classes of the contexts (computed on first use)
     // second stream of the learn launches (kernels of independent width
     // classes run side by side), its fork and join events; created on first use
@@ -341,6 +343,8 @@ struct f2_store {
     int* counters;
     int* plan_hist;         // key histogram / cursors of the plan kernels
     int32_t* rep_count;     // representatives per context (pass 1 output)
+    int32_t* shard_reps;    // [8C]: representatives of each shard of a split context (pass 1)
+    int32_t* shard_done;    // [C]: finished shards of a split context
     int32_t* rep_list;      // per-row scratch of pass 1 (capacity rep_capacity rows)
     int32_t* rep_dup;
     int64_t rep_capacity;
@@ -402,10 +406,33 @@ constexpr int64_t DEFAULT_HOST_CHUNK_BYTES = int64_t(512) << 20;
 // Host helpers (store.cu, encode.cu, host_io.cu).
 void f2_host_io_free(f2_store* st);
 int f2_cuda_status(cudaError_t e);
+// Queue slots beyond one per context, for the shard items of split contexts.
+inline int f2_shard_queue_extra(int num_sms) { return 16 * num_sms + 64; }
+
 // Every device allocation made by a call on a store goes through here (the
 // stream-ordered allocator with a stream, cudaMalloc without one), so the
 // F2_OPT_FAIL_ALLOC hook can make it fail.
 cudaError_t f2_dev_alloc(const f2_store* st, void** p, size_t bytes, cudaStream_t cs, bool stream_ordered);
+// Byte fills of several device buffers in one kernel launch (what a call
+// would otherwise spend one memset node on each); null or empty segments
+// are skipped.
+struct F2FillList {
+    static constexpr int MAX = 12;
+    void* p[MAX];
+    unsigned long long bytes[MAX];
+    unsigned int value[MAX];  // byte value
+    int n = 0;
+    void add(void* ptr, size_t nbytes, unsigned int byte = 0)
+    {
+        if (ptr && nbytes && n < MAX) {
+            p[n] = ptr;
+            bytes[n] = nbytes;
+            value[n] = byte & 0xffu;
+            ++n;
+        }
+    }
+};
+cudaError_t f2_fill(const F2FillList& L, cudaStream_t cs);
 int f2_ensure_aux(const f2_store* st);  // second stream and fork/join events, created on first use
 int f2_encode_table_min_default();
 int f2_encode_table_min_floor();

@@ -79,6 +79,8 @@ struct DedupArgs {
     const int32_t* queue;
     int* counters;
     unsigned long long* timing;  // per-context timestamps (F2_OPT_TIMING), NULL = off
+    int32_t* shard_reps;         // [DD_MAX_SHARDS * C]: representatives of each shard of a split context
+    int32_t* shard_done;         // [C]: shards of a split context finished (the last one compacts)
 };
 
 // Per-context timestamps of a learn call (diagnostics, F2_OPT_TIMING):
@@ -131,6 +133,28 @@ constexpr int DD_K = 2;                         // rows per thread per round (fe
 constexpr int DD_XW = NARROW_WD;                // widest feature row (words) of dedup_kernel<false>
 constexpr int DD_XW_WIDE = 16;                  // widest of dedup_kernel<true> (one row in flight)
 constexpr int DEDUP_PROBES = 8;                 // linear-probe limit
+// A CTA-owned context with much more than its share of the call's rows is
+// split into up to DD_MAX_SHARDS consecutive row ranges deduplicated by
+// different CTAs (a queue item = context | shard << 24 | (shards - 1) << 28).
+constexpr int DD_MAX_SHARDS = 8;
+constexpr int SHARD_CTX_LIMIT = 1 << 24;
+// Shards of at most this many rows (a shard's table of DD_CTA_E entries
+// stays at most half full when half its rows repeat earlier ones).
+#ifndef F2_DD_SHARD_ROWS
+#define F2_DD_SHARD_ROWS 16384
+#endif
+constexpr int DD_SHARD_ROWS = F2_DD_SHARD_ROWS;
+// A context of the 4-warp class with more than 1/DD_QUAD_SHARE of a shard
+// share goes to a whole CTA (4 warps would finish it long after the SMs'
+// median).
+#ifndef F2_DD_QUAD_PROMOTE
+#define F2_DD_QUAD_PROMOTE 1
+#endif
+constexpr int DD_QUAD_SHARE = 4;
+// Neither applies below these sizes, where a CTA's fixed costs (its table,
+// its barriers, the shards' compaction) outweigh what the split saves.
+constexpr int DD_PROMOTE_MIN_ROWS = 1024;
+constexpr int DD_SHARD_MIN_ROWS = 2048;
 static_assert(DD_WARPS * DD_WARP_REGION * 4 <= DD_SMEM, "warp regions exceed the dedup shared memory");
 
 __host__ __device__ __forceinline__ int elim_words(int d, int wd) { return CTL_WORDS + d * row_stride(wd); }
@@ -336,9 +360,30 @@ __device__ __forceinline__ void dd_sync()
 // takes DD_K rows a round (one for feature rows of 3 or more words).  Table slot: (fingerprint, smallest row index
 // of that content) plus a duplicate counter; a full row comparison decides
 // every match, so a row is a duplicate only if it equals an earlier row.
+//
+// Shard k of nsh takes the context's rows [lo, hi) = [T*k/nsh, T*(k+1)/nsh)
+// and writes its representatives, numbered from lo, at
+// rep_list[row_off[c] + lo + ...]; a row
+// equal to a row of an earlier shard becomes its own representative there,
+// which the elimination classifies exactly all the same (it lies in the span
+// when it arrives).  The last shard to finish moves the shards' lists
+// together, in stream order, and sets rep_count[c].  Returns whether the
+// context is done (false in the shards that did not finish last).
+//
+// The queue item of the context a dedup CTA is on (context, shard, shard
+// count); a CTA-owned pass reads it here, before and again after its rows, so
+// that no register holds it through them.
+__shared__ uint32_t dd_cta_item;
+
 template <int G, int XW>
-__device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t* region, int E, int* wcnt)
+__device__ bool dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t* region, int E, int* wcnt)
 {
+    int shard = 0, nsh = 1;
+    if constexpr (G == DD_WARPS) {
+        const uint32_t qi = dd_cta_item;
+        shard = (int)((qi >> 24) & 7u);
+        nsh = (int)(qi >> 28) + 1;
+    }
     constexpr int NT = 32 * G;
     const int lane = threadIdx.x & 31;
     const int gw = (G == 1) ? 0 : (int)((threadIdx.x >> 5) % G);  // warp within the group
@@ -347,9 +392,11 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
     int* D = reinterpret_cast<int*>(region + 2 * E);
     const CtxDesc cd = s.desc[c];
     const int n = cd.n;
-    const int64_t r0 = a.row_off[c];
-    const int T = (int)(a.row_off[c + 1] - r0);
-    const uint32_t* xc = a.x + a.x_off[c];
+    const int Tc = (int)(a.row_off[c + 1] - a.row_off[c]);
+    const int lo = (int)(((long long)Tc * shard) / nsh);
+    const int64_t r0 = a.row_off[c] + lo;  // this shard's rows, and its part of rep_list / rep_dup
+    const int T = (int)(((long long)Tc * (shard + 1)) / nsh) - lo;
+    const uint32_t* xc = a.x + a.x_off[c] + (int64_t)lo * XW;
     const uint4* yc = a.y + r0;
     const uint32_t lm = last_mask(n);
     const uint32_t emask = (uint32_t)(E - 1);
@@ -477,7 +524,7 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
             }
             if ((bal[j] >> lane) & 1u) {
                 const int pos = nrep + before + __popc(bal[j] & ((1u << lane) - 1u));
-                a.rep_list[r0 + pos] = base + j * NT + t;
+                a.rep_list[r0 + pos] = base + j * NT + t;  // within the shard (see below)
                 a.rep_dup[r0 + pos] = mine[j];
             }
             nrep += total;
@@ -490,13 +537,63 @@ __device__ void dedup_ctx(const StoreDev& s, const DedupArgs& a, int c, uint32_t
         a.rep_dup[r0 + k] = (slot >= 0) ? D[slot] : 0;
     }
     if (t == 0) {
-        a.rep_count[c] = nrep;
         // the call's work, for the elimination plan's thresholds
         atomicAdd(reinterpret_cast<unsigned long long*>(a.counters + CNT_WORK),
                   (unsigned long long)nrep * (unsigned long long)cd.d);
         atomicAdd(reinterpret_cast<unsigned long long*>(a.counters + CNT_REPS), (unsigned long long)nrep);
     }
+    if constexpr (G == DD_WARPS) {
+        const uint32_t qi = *reinterpret_cast<const volatile uint32_t*>(&dd_cta_item);
+        shard = (int)((qi >> 24) & 7u);
+        nsh = (int)(qi >> 28) + 1;
+    }
+    if (nsh == 1) {
+        if (t == 0) a.rep_count[c] = nrep;
+        dd_sync<G>();
+        return true;
+    }
+    // a split context: publish this shard's count; the last shard to finish
+    // moves the lists of shards 1.. down behind shard 0's (never upward: a
+    // shard's list starts at or after its destination), chunk by chunk
+    // through registers, renumbering their rows from the context's first
+    __shared__ int s_last;
+    __threadfence();  // this thread's list entries, before the count that publishes them
     dd_sync<G>();
+    if (t == 0) {
+        a.shard_reps[(size_t)DD_MAX_SHARDS * c + shard] = nrep;
+        __threadfence();
+        s_last = (atomicAdd(a.shard_done + c, 1) == nsh - 1);
+    }
+    dd_sync<G>();
+    if (!s_last) return false;
+    __threadfence();
+    const int64_t cbase = a.row_off[c];
+    const int Tall = (int)(a.row_off[c + 1] - cbase);
+    int dst = 0;
+    for (int k = 0; k < nsh; ++k) {
+        const int src = (int)(((long long)Tall * k) / nsh);
+        const int cnt = __ldcg(a.shard_reps + (size_t)DD_MAX_SHARDS * c + k);
+        if (k > 0) {
+            for (int b0 = 0; b0 < cnt; b0 += NT) {
+                const int j = b0 + t;
+                int32_t rl = 0, rd = 0;
+                if (j < cnt) {
+                    rl = __ldcg(a.rep_list + cbase + src + j) + src;
+                    rd = __ldcg(a.rep_dup + cbase + src + j);
+                }
+                dd_sync<G>();
+                if (j < cnt) {
+                    a.rep_list[cbase + dst + j] = rl;
+                    a.rep_dup[cbase + dst + j] = rd;
+                }
+                dd_sync<G>();
+            }
+        }
+        dst += cnt;
+    }
+    if (t == 0) a.rep_count[c] = dst;
+    dd_sync<G>();
+    return true;
 }
 
 __device__ __forceinline__ int pow2_at_least(int v)
@@ -523,23 +620,31 @@ __global__ void __launch_bounds__(DD_THREADS, DD_CTAS_PER_SM) dedup_kernel(Store
         const int b = a.counters[CNT_BEGIN + C_CTA];
         for (;;) {
             __syncthreads();
-            if (threadIdx.x == 0) s_item[0] = atomicAdd(a.counters + CNT_HEAD + C_CTA, 1);
+            if (threadIdx.x == 0) {
+                const int it = atomicAdd(a.counters + CNT_HEAD + C_CTA, 1);
+                s_item[0] = it;
+                if (it < n) dd_cta_item = (uint32_t)a.queue[b + it];
+            }
             __syncthreads();
             const int item = s_item[0];
             if (item >= n) break;
-            const int c = a.queue[b + item];
+            const uint32_t qi = dd_cta_item;
+            const int c = (int)(qi & (SHARD_CTX_LIMIT - 1));
+            const int nsh = (int)(qi >> 28) + 1;
             const int T = (int)(a.row_off[c + 1] - a.row_off[c]);
-            int E = pow2_at_least(2 * T);
+            int E = pow2_at_least(2 * ((T + nsh - 1) / nsh));
             if (E > DD_CTA_E) E = DD_CTA_E;
-            if (threadIdx.x == 0) time_mark(a.timing, c, 0);
-#define F2_DD_CTA(W) dedup_ctx<DD_WARPS, W>(s, a, c, smem, E, wcnt)
+            // a split context's pass: from its first shard's start to the end of the last one
+            if (threadIdx.x == 0 && ((qi >> 24) & 7u) == 0) time_mark(a.timing, c, 0);
+            bool done = true;
+#define F2_DD_CTA(W) done = dedup_ctx<DD_WARPS, W>(s, a, c, smem, E, wcnt)
             if constexpr (WX) {
                 F2_XWIDE_SWITCH(s.desc[c].xw, F2_DD_CTA)
             } else {
                 F2_NARROW_SWITCH(s.desc[c].xw, F2_DD_CTA)
             }
 #undef F2_DD_CTA
-            if (threadIdx.x == 0) time_mark(a.timing, c, 1);
+            if (threadIdx.x == 0 && done) time_mark(a.timing, c, 1);
         }
     }
     {
@@ -1312,97 +1417,143 @@ struct PlanArgs {
     int64_t warp_work;
     int scale;     // mode 1: scale heavy_rows / warp_work to the totals of the duplicate pass
     int num_sms;
+    long long shard_work;  // mode 0: rows x (xw + 4) of one shard share; 0 = no splitting
+    int max_shards;        // mode 0: most shards of one context
+    int shard_cap;         // mode 0: queue slots for shard items beyond one per context
     int32_t* queue;
     int32_t* keybuf;
     int* hist;     // PLAN_KEYS counts (zeroed before plan_key_kernel), then cursors
+    int hist_zeroed;  // hist is zero already (else launch_plan clears it)
     int* counters;
 };
+
+// Ownership thresholds of the elimination plan, scaled to the call's work
+// when the duplicate pass has measured it: a warp-owned context must not run
+// (dependent round after round) much longer than the whole call.
+struct PlanLimits {
+    long long heavy_rows, warp_work;
+};
+__device__ __forceinline__ PlanLimits plan_limits(const PlanArgs& p)
+{
+    PlanLimits L{p.heavy_rows, p.warp_work};
+    if (p.mode == 1 && p.scale) {
+        const unsigned long long tw = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_WORK);
+        const unsigned long long tr = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_REPS);
+        const long long hr = (long long)(tr / ((unsigned long long)p.num_sms * HEAVY_REPS_DIV));
+        const long long ww = (long long)(tw / ((unsigned long long)p.num_sms * WARP_WORK_DIV));
+        L.heavy_rows = hr < HEAVY_ROWS_MIN ? HEAVY_ROWS_MIN : (hr > L.heavy_rows ? L.heavy_rows : hr);
+        L.warp_work = ww < WARP_WORK_MIN ? WARP_WORK_MIN : (ww > L.warp_work ? L.warp_work : ww);
+    }
+    return L;
+}
+
+// Validates context c's part of the batch and returns its key (bits 0..15:
+// class, work bucket and width; bits 16..18: shards - 1), or -1 when it has
+// no work; nsh_out = its queue items.
+__device__ __forceinline__ int plan_key_of(const StoreDev& s, const PlanArgs& p, const PlanLimits& L, int c,
+                                           int& nsh_out)
+{
+    nsh_out = 0;
+    const CtxDesc cd = s.desc[c];
+    int64_t R;
+    if (p.mode == 1 && p.rep_count) {
+        R = p.rep_count[c];
+        if (R <= -2) R = -(R + 2);
+    } else {
+        const int64_t a0 = p.row_off[c], a1 = p.row_off[c + 1];
+        const int64_t rows = a1 - a0;
+        const int64_t x0 = p.x_off[c];
+        const bool ok = a0 >= 0 && rows >= 0 && rows < (1ll << 31) && a1 <= p.total_rows && x0 >= 0 &&
+                        rows <= p.total_xw && x0 + rows * cd.xw <= p.total_xw;
+        if (!ok) record_status(s.status, F2_ERR_ROWS);
+        R = ok ? rows : -1;
+        if (p.mode == 0 && p.rep_count) {
+            // wide rows are not deduplicated; rows of a full-rank context
+            // are checked one by one (verify_full_kernel)
+            if (R > 0 && (cd.xw > DD_XW_WIDE || s.rank[c] == cd.d)) {
+                p.rep_count[c] = (int32_t)(-(R + 2));
+                R = 0;
+            } else {
+                p.rep_count[c] = (R > 0) ? 0 : (int32_t)R;
+            }
+        }
+    }
+    int key = -1;
+    if (R > 0) {
+        int cls;
+        unsigned long long work;
+        if (p.mode == 0) {
+            cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : (R <= DD_QUAD_MAX_ROWS ? CLS_DD_QUAD : CLS_DD_CTA);
+            if (cd.xw > DD_XW) cls += CLS_DDW_CTA - CLS_DD_CTA;  // the 10..16-word instance
+            work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
+        } else {
+            const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= L.heavy_rows ||
+                               R * cd.d > L.warp_work;
+            if (s.rank[c] == cd.d) cls = CLS_FULL;
+            else if (cd.wd > NARROW_WD) cls = (cd.wd <= WIDE_M_WD) ? CLS_WIDE_M : CLS_WIDE;
+            else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
+            else cls = heavy ? CLS_CTA : CLS_WARP;
+            work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
+        }
+        int nsh = 1;
+        if (p.mode == 0 && p.shard_work > 0) {
+            if (F2_DD_QUAD_PROMOTE && (cls == CLS_DD_QUAD || cls == CLS_DDW_QUAD) && R >= DD_PROMOTE_MIN_ROWS &&
+                (long long)work * DD_QUAD_SHARE > p.shard_work)
+                cls += CLS_DD_CTA - CLS_DD_QUAD;
+            if (cls == CLS_DD_CTA || cls == CLS_DDW_CTA) {
+                long long k = (long long)work / p.shard_work;
+                if (DD_SHARD_ROWS > 0 && (R + DD_SHARD_ROWS - 1) / DD_SHARD_ROWS > k)
+                    k = (R + DD_SHARD_ROWS - 1) / DD_SHARD_ROWS;
+                if (k > R / DD_SHARD_MIN_ROWS) k = R / DD_SHARD_MIN_ROWS;
+                nsh = k < 1 ? 1 : (k > p.max_shards ? p.max_shards : (int)k);
+                // the queue holds shard_cap extra items; past that, contexts stay whole
+                if (nsh > 1 && atomicAdd(p.counters + CNT_SHARDS, nsh - 1) + (nsh - 1) > p.shard_cap) nsh = 1;
+                work /= (unsigned long long)nsh;
+            }
+        }
+        int bucket = 63 - __clzll(work);
+        if (bucket >= PLAN_BUCKETS) bucket = PLAN_BUCKETS - 1;
+        const int width = (p.mode == 0 ? cd.xw : cd.wd);
+        const int sub = (PLAN_BUCKETS - 1 - bucket) * NARROW_WD + (width > NARROW_WD ? NARROW_WD : width) - 1;
+        key = cls * PLAN_SUB + sub;
+        key |= (nsh - 1) << 16;
+        nsh_out = nsh;
+    }
+    return key;
+}
 
 __global__ void __launch_bounds__(256) plan_key_kernel(StoreDev s, PlanArgs p)
 {
     __shared__ int hist[PLAN_KEYS];
     for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    // ownership thresholds, scaled to the call's work when the duplicate
-    // pass has measured it: a warp-owned context must not run (dependent
-    // round after round) much longer than the whole call
-    long long heavy_rows = p.heavy_rows, warp_work = p.warp_work;
-    if (p.mode == 1 && p.scale) {
-        const unsigned long long tw = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_WORK);
-        const unsigned long long tr = *reinterpret_cast<const unsigned long long*>(p.counters + CNT_REPS);
-        const long long hr = (long long)(tr / ((unsigned long long)p.num_sms * HEAVY_REPS_DIV));
-        const long long ww = (long long)(tw / ((unsigned long long)p.num_sms * WARP_WORK_DIV));
-        heavy_rows = hr < HEAVY_ROWS_MIN ? HEAVY_ROWS_MIN : (hr > heavy_rows ? heavy_rows : hr);
-        warp_work = ww < WARP_WORK_MIN ? WARP_WORK_MIN : (ww > warp_work ? warp_work : ww);
-    }
+    const PlanLimits L = plan_limits(p);
     for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
-        const CtxDesc cd = s.desc[c];
-        int64_t R;
-        if (p.mode == 1 && p.rep_count) {
-            R = p.rep_count[c];
-            if (R <= -2) R = -(R + 2);
-        } else {
-            const int64_t a0 = p.row_off[c], a1 = p.row_off[c + 1];
-            const int64_t rows = a1 - a0;
-            const int64_t x0 = p.x_off[c];
-            const bool ok = a0 >= 0 && rows >= 0 && rows < (1ll << 31) && a1 <= p.total_rows && x0 >= 0 &&
-                            rows <= p.total_xw && x0 + rows * cd.xw <= p.total_xw;
-            if (!ok) record_status(s.status, F2_ERR_ROWS);
-            R = ok ? rows : -1;
-            if (p.mode == 0 && p.rep_count) {
-                // wide rows are not deduplicated; rows of a full-rank context
-                // are checked one by one (verify_full_kernel)
-                if (R > 0 && (cd.xw > DD_XW_WIDE || s.rank[c] == cd.d)) {
-                    p.rep_count[c] = (int32_t)(-(R + 2));
-                    R = 0;
-                } else {
-                    p.rep_count[c] = (R > 0) ? 0 : (int32_t)R;
-                }
-            }
-        }
-        int key = -1;
-        if (R > 0) {
-            int cls;
-            unsigned long long work;
-            if (p.mode == 0) {
-                cls = (R <= DD_WARP_MAX_ROWS) ? CLS_DD_WARP : (R <= DD_QUAD_MAX_ROWS ? CLS_DD_QUAD : CLS_DD_CTA);
-                if (cd.xw > DD_XW) cls += CLS_DDW_CTA - CLS_DD_CTA;  // the 10..16-word instance
-                work = (unsigned long long)R * (unsigned long long)(cd.xw + 4);
-            } else {
-                const bool heavy = elim_words(cd.d, cd.wd) > p.warp_region_words || R >= heavy_rows ||
-                                   R * cd.d > warp_work;
-                if (s.rank[c] == cd.d) cls = CLS_FULL;
-                else if (cd.wd > NARROW_WD) cls = (cd.wd <= WIDE_M_WD) ? CLS_WIDE_M : CLS_WIDE;
-                else if (cd.wd <= SMALL_WD) cls = heavy ? CLS_CTA_S : CLS_WARP_S;
-                else cls = heavy ? CLS_CTA : CLS_WARP;
-                work = (unsigned long long)R * (unsigned long long)(cd.wd + 4) * (unsigned long long)cd.d;
-            }
-            int bucket = 63 - __clzll(work);
-            if (bucket >= PLAN_BUCKETS) bucket = PLAN_BUCKETS - 1;
-            const int width = (p.mode == 0 ? cd.xw : cd.wd);
-            const int sub = (PLAN_BUCKETS - 1 - bucket) * NARROW_WD + (width > NARROW_WD ? NARROW_WD : width) - 1;
-            key = cls * PLAN_SUB + sub;
-            atomicAdd(&hist[key], 1);
-        }
-        p.keybuf[c] = key;
+        int nsh;
+        const int kv = plan_key_of(s, p, L, c, nsh);
+        if (kv >= 0) atomicAdd(&hist[kv & 0xFFFF], nsh);
+        p.keybuf[c] = kv;
     }
     __syncthreads();
     for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x)
         if (hist[i]) atomicAdd(p.hist + i, hist[i]);
 }
 
-// Exclusive scan of the key counts in key order (one block of 1024).
-__global__ void __launch_bounds__(1024) plan_scan_kernel(PlanArgs p)
+// Exclusive scan of the key counts `hist` (global or shared) in key order by
+// one block of 1024 threads; hist becomes the cursors and the class blocks of
+// `counters` (first item, count, head) are set.
+__device__ void plan_scan_block(int* hist, int* counters)
 {
     constexpr int PER = (PLAN_KEYS + 1023) / 1024;
     __shared__ int wsum[32];
+    __shared__ int s_total;
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     int v[PER];
     int tot = 0;
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
         const int k = t * PER + j;
-        v[j] = (k < PLAN_KEYS) ? p.hist[k] : 0;
+        v[j] = (k < PLAN_KEYS) ? hist[k] : 0;
         tot += v[j];
     }
     int inc = tot;
@@ -1422,40 +1573,85 @@ __global__ void __launch_bounds__(1024) plan_scan_kernel(PlanArgs p)
             if (lane >= o) wi += u;
         }
         wsum[lane] = wi - w;
+        if (lane == 31) s_total = wi;
     }
     __syncthreads();
     int run = wsum[warp] + inc - tot;
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
         const int k = t * PER + j;
-        if (k < PLAN_KEYS) {
-            p.hist[k] = run;  // becomes the cursor of key k
-            if (k % PLAN_SUB == 0) {
-                const int cls = k / PLAN_SUB;
-                p.counters[CNT_BEGIN + cls] = run;
-                p.counters[CNT_HEAD + cls] = 0;
-            }
-            run += v[j];
-            if (k % PLAN_SUB == PLAN_SUB - 1) {
-                const int cls = k / PLAN_SUB;
-                p.counters[CNT_COUNT + cls] = run - p.counters[CNT_BEGIN + cls];
-            }
-        }
+        if (k < PLAN_KEYS) hist[k] = run;  // becomes the cursor of key k
+        run += v[j];
+    }
+    __syncthreads();
+    // a class's items run from the cursor of its first key to that of the next class
+    if (t < NUM_CLASSES) {
+        const int b = hist[t * PLAN_SUB];
+        const int e = (t + 1 < NUM_CLASSES) ? hist[(t + 1) * PLAN_SUB] : s_total;
+        counters[CNT_BEGIN + t] = b;
+        counters[CNT_HEAD + t] = 0;
+        counters[CNT_COUNT + t] = e - b;
+    }
+}
+
+__global__ void __launch_bounds__(1024) plan_scan_kernel(PlanArgs p) { plan_scan_block(p.hist, p.counters); }
+
+// Queue item(s) of context c with key kv at the cursor of its key.
+__device__ __forceinline__ void plan_place(const PlanArgs& p, int* cursor, int c, int kv)
+{
+    const int key = kv & 0xFFFF, nsh = (kv >> 16) + 1;
+    if (nsh == 1) {
+        p.queue[atomicAdd(cursor + key, 1)] = c;
+    } else {  // one item per shard
+        const int q0 = atomicAdd(cursor + key, nsh);
+        for (int k = 0; k < nsh; ++k)
+            p.queue[q0 + k] = (int32_t)((uint32_t)c | ((uint32_t)k << 24) | ((uint32_t)(nsh - 1) << 28));
     }
 }
 
 __global__ void __launch_bounds__(256) plan_scatter_kernel(StoreDev s, PlanArgs p)
 {
     for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
-        const int key = p.keybuf[c];
-        if (key >= 0) p.queue[atomicAdd(p.hist + key, 1)] = c;
+        const int kv = p.keybuf[c];
+        if (kv >= 0) plan_place(p, p.hist, c, kv);
+    }
+}
+
+// The three steps in one block, the histogram in shared memory, for stores
+// of at most PLAN_SMALL_MAX contexts (one launch instead of a memset and
+// three kernels: what a small batch waits for).
+constexpr int PLAN_SMALL_MAX = 8192;
+__global__ void __launch_bounds__(1024) plan_small_kernel(StoreDev s, PlanArgs p)
+{
+    __shared__ int hist[PLAN_KEYS];
+    for (int i = threadIdx.x; i < PLAN_KEYS; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    const PlanLimits L = plan_limits(p);
+    for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
+        int nsh;
+        const int kv = plan_key_of(s, p, L, c, nsh);
+        if (kv >= 0) atomicAdd(&hist[kv & 0xFFFF], nsh);
+        p.keybuf[c] = kv;  // read back below by this same thread
+    }
+    __syncthreads();
+    plan_scan_block(hist, p.counters);
+    __syncthreads();
+    for (int c = threadIdx.x; c < s.num_ctx; c += blockDim.x) {
+        const int kv = p.keybuf[c];
+        if (kv >= 0) plan_place(p, hist, c, kv);
     }
 }
 
 int launch_plan(const StoreDev& sd, const PlanArgs& pa, int num_sms, cudaStream_t cs)
 {
-    cudaError_t e = cudaMemsetAsync(pa.hist, 0, sizeof(int) * PLAN_KEYS, cs);
-    if (e != cudaSuccess) return f2_cuda_status(e);
+    if (sd.num_ctx <= PLAN_SMALL_MAX) {
+        plan_small_kernel<<<1, 1024, 0, cs>>>(sd, pa);
+        return f2_cuda_status(cudaGetLastError());
+    }
+    if (!pa.hist_zeroed) {
+        const cudaError_t e = cudaMemsetAsync(pa.hist, 0, sizeof(int) * PLAN_KEYS, cs);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
     int blocks = (sd.num_ctx + 255) / 256;
     if (blocks > num_sms * 2) blocks = num_sms * 2;
     if (blocks < 1) blocks = 1;
@@ -1708,17 +1904,22 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
                        int64_t total_rows, int64_t total_xw, int32_t* rep_count, int64_t heavy_rows,
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
-                       unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr, int scale = 0)
+                       unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr, int scale = 0,
+                       bool prezeroed = false)
 {
+    // prezeroed: the caller has cleared full_ctr's first 2C words and late
+    // count, full_cnt, full_first (to -1) and hist
     // full_ctr: chunks claimed [C], chunks done [C], late start [C], late list [C], late count
     const int C = sd.num_ctx;
     LearnArgs lx = la;
     lx.late_start = full_ctr + 2 * C;
     lx.late_list = full_ctr + 3 * C;
     lx.late_count = full_ctr + 4 * C;
-    {
+    if (!prezeroed) {
         cudaError_t e0 = cudaMemsetAsync(full_ctr, 0, sizeof(int) * 2 * (size_t)C, cs);
         if (e0 == cudaSuccess) e0 = cudaMemsetAsync(lx.late_count, 0, sizeof(int), cs);
+        if (e0 == cudaSuccess) e0 = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
+        if (e0 == cudaSuccess) e0 = cudaMemsetAsync(full_first, 0xff, sizeof(unsigned long long) * (size_t)C, cs);
         if (e0 != cudaSuccess) return f2_cuda_status(e0);
     }
     PlanArgs pa;
@@ -1733,9 +1934,13 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     pa.warp_work = warp_work;
     pa.scale = scale;
     pa.num_sms = num_sms;
+    pa.shard_work = 0;
+    pa.max_shards = 1;
+    pa.shard_cap = 0;
     pa.queue = queue;
     pa.keybuf = keybuf;
     pa.hist = hist;
+    pa.hist_zeroed = prezeroed;
     pa.counters = la.counters;
     int rc = launch_plan(sd, pa, num_sms, cs);
     if (rc != F2_OK) return rc;
@@ -1780,6 +1985,8 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         rc = wide(elim_wide_kernel<WIDE_M_WD, CLS_WIDE_M>, wv.max_wide_m_d, WIDE_M_WD);
         if (rc != F2_OK) return rc;
     }
+    const size_t small_words = (size_t)LEARN_WARPS * (size_t)la.small_region_words;
+    const size_t small_smem = 4 * (small_words > (size_t)wv.max_small_words ? small_words : (size_t)wv.max_small_words);
     if (wv.has_narrow) {
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
@@ -1787,20 +1994,15 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         if (rc != F2_OK) return rc;
     }
     if (wv.has_small) {
-        const size_t words = (size_t)LEARN_WARPS * (size_t)la.small_region_words;
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
-        rc = narrow(elim_narrow_kernel<true>,
-                    4 * (words > (size_t)wv.max_small_words ? words : (size_t)wv.max_small_words), ks);
+        rc = narrow(elim_narrow_kernel<true>, small_smem, ks);
         if (rc != F2_OK) return rc;
     }
     e = f.join();
     if (e != cudaSuccess) return f2_cuda_status(e);
     {  // full-rank contexts: at the start of the call (the plan decides on the
        // device which, if any) or reached during it (listed by the kernels above)
-        e = cudaMemsetAsync(full_cnt, 0, sizeof(unsigned long long) * (size_t)C, cs);
-        if (e == cudaSuccess) e = cudaMemsetAsync(full_first, 0xff, sizeof(unsigned long long) * (size_t)C, cs);
-        if (e != cudaSuccess) return f2_cuda_status(e);
         FullArgs fa;
         fa.row_off = row_off;
         fa.x_off = x_off;
@@ -1880,12 +2082,26 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (e != cudaSuccess) return F2_ERR_OOM;
         st->rep_capacity = total_rows;
     }
+    // every scratch counter of the call, zeroed by one launch
+    const size_t C = (size_t)st->num_ctx;
+    F2FillList zl;
     if (st->timing_on) {  // diagnostics: per-context timestamps of this call
-        const size_t bytes = sizeof(unsigned long long) * TIME_WORDS * (size_t)(st->num_ctx > 0 ? st->num_ctx : 1);
+        const size_t bytes = sizeof(unsigned long long) * TIME_WORDS * C;
         if (!st->timing && f2_dev_alloc(st, (void**)&st->timing, bytes, cs, true) != cudaSuccess) return F2_ERR_OOM;
-        e = cudaMemsetAsync(st->timing, 0, bytes, cs);
-        if (e != cudaSuccess) return f2_cuda_status(e);
+        zl.add(st->timing, bytes);
     }
+    if (dedup) {  // the work totals and the shard items of the duplicate pass
+        zl.add(st->counters + CNT_WORK, (CNT_WORDS - CNT_WORK) * sizeof(int));
+        zl.add(st->shard_done, sizeof(int32_t) * C);
+    }
+    zl.add(st->full_ctr, sizeof(int) * 2 * C);        // full-rank chunks claimed and done
+    zl.add(st->full_ctr + 4 * C, sizeof(int));        // late count
+    zl.add(st->full_cnt, sizeof(unsigned long long) * C);
+    zl.add(st->full_first, sizeof(unsigned long long) * C, 0xff);
+    if (st->num_ctx > PLAN_SMALL_MAX)  // the histograms of the two plans (one block keeps its own)
+        zl.add(st->plan_hist, sizeof(int) * 2 * PLAN_HIST_WORDS);
+    e = f2_fill(zl, cs);
+    if (e != cudaSuccess) return f2_cuda_status(e);
     const StoreDev sd = st->dev();
     {
         const int rc = f2_ensure_aux(st);
@@ -1893,8 +2109,6 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     Fork fk{cs, st->aux, st->ev_fork, st->ev_join};
     if (dedup) {
-        e = cudaMemsetAsync(st->counters + CNT_WORK, 0, 4 * sizeof(int), cs);  // the work totals
-        if (e != cudaSuccess) return f2_cuda_status(e);
         PlanArgs pa;
         pa.row_off = row_off;
         pa.x_off = x_off;
@@ -1907,9 +2121,16 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         pa.warp_work = 0;
         pa.scale = 0;
         pa.num_sms = st->num_sms;
+        // a shard share: the call's rows x (feature words + 4) over four per SM
+        pa.max_shards = st->dd_shards;
+        pa.shard_cap = f2_shard_queue_extra(st->num_sms);
+        pa.shard_work = (st->num_ctx < SHARD_CTX_LIMIT && st->dd_shards > 1)
+                            ? (total_x_words + 4 * total_rows) / (4 * (long long)st->num_sms) + 1
+                            : 0;
         pa.queue = st->queue;
         pa.keybuf = st->keybuf;
         pa.hist = st->plan_hist;
+        pa.hist_zeroed = 1;
         pa.counters = st->counters;
         int rc = launch_plan(sd, pa, st->num_sms, cs);
         if (rc != F2_OK) return rc;
@@ -1924,6 +2145,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         da.queue = st->queue;
         da.counters = st->counters;
         da.timing = st->timing_on ? st->timing : nullptr;
+        da.shard_reps = st->shard_reps;
+        da.shard_done = st->shard_done;
         // the two instances hold disjoint contexts: side by side when both run
         const bool wide_rows = st->max_xw > DD_XW;  // some context has feature rows of 10..16 words
         e = cudaFuncSetAttribute(dedup_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
@@ -1936,7 +2159,7 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (wide_rows) {
             e = cudaFuncSetAttribute(dedup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, DD_SMEM);
             if (e != cudaSuccess) return f2_cuda_status(e);
-            dedup_kernel<true><<<DD_CTAS_PER_SM * st->num_sms, DD_THREADS, DD_SMEM, cs>>>(sd, da);
+            dedup_kernel<true><<<DD_CTAS_PER_SM * st->num_sms, DD_THREADS, DD_SMEM, fk.next(1)>>>(sd, da);
             e = cudaGetLastError();
             if (e != cudaSuccess) return f2_cuda_status(e);
         }
@@ -1975,8 +2198,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     const int scale = dedup && !st->heavy_rows_set && !st->warp_work_set;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
-                              heavy, st->warp_work, st->queue, st->keybuf, st->plan_hist, st->num_sms, wv,
-                              st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale);
+                              heavy, st->warp_work, st->queue, st->keybuf, st->plan_hist + PLAN_HIST_WORDS,
+                              st->num_sms, wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale, true);
 }
 
 extern "C" int f2_learn_timing(const f2_store* st, uint64_t* out_host, f2_stream_t stream)

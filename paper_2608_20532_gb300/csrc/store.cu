@@ -30,6 +30,44 @@ cudaError_t f2_dev_alloc(const f2_store* st, void** p, size_t bytes, cudaStream_
     return stream_ordered ? cudaMallocAsync(p, bytes, cs) : cudaMalloc(p, bytes);
 }
 
+namespace {
+
+// Grid-stride byte fill of each segment: 16-byte stores between the
+// segment's aligned head and tail, single bytes at both ends.
+__global__ void __launch_bounds__(256) fill_kernel(F2FillList L)
+{
+    const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const size_t nth = (size_t)gridDim.x * blockDim.x;
+    for (int k = 0; k < L.n; ++k) {
+        uint8_t* p = static_cast<uint8_t*>(L.p[k]);
+        const size_t bytes = L.bytes[k];
+        const uint8_t b = (uint8_t)L.value[k];
+        const uint32_t w = 0x01010101u * b;
+        size_t head = (16 - ((uintptr_t)p & 15)) & 15;
+        if (head > bytes) head = bytes;
+        const size_t n16 = (bytes - head) / 16;
+        for (size_t i = tid; i < head; i += nth) p[i] = b;
+        uint4* q = reinterpret_cast<uint4*>(p + head);
+        for (size_t i = tid; i < n16; i += nth) q[i] = make_uint4(w, w, w, w);
+        for (size_t i = head + 16 * n16 + tid; i < bytes; i += nth) p[i] = b;
+    }
+}
+
+}  // namespace
+
+cudaError_t f2_fill(const F2FillList& L, cudaStream_t cs)
+{
+    if (L.n == 0) return cudaSuccess;
+    unsigned long long total = 0;
+    for (int k = 0; k < L.n; ++k) total += L.bytes[k];
+    // about 16 KB a block, at most 1024 blocks
+    unsigned long long blocks = (total + 16383) / 16384;
+    if (blocks > 1024) blocks = 1024;
+    if (blocks < 1) blocks = 1;
+    fill_kernel<<<(unsigned)blocks, 256, 0, cs>>>(L);
+    return cudaGetLastError();
+}
+
 int f2_ensure_aux(const f2_store* st)
 {
     if (st->aux) return F2_OK;
@@ -74,7 +112,7 @@ static void free_store(f2_store* s)
     if (s->ev_join) cudaEventDestroy(s->ev_join);
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
-                    s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup,
+                    s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup, s->shard_reps, s->shard_done,
                     s->full_ctr, s->full_cnt, s->full_first,
                     s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items, s->enc_hot, s->enc_tab_off,
                     s->enc_pool, s->timing};
@@ -85,21 +123,17 @@ static void free_store(f2_store* s)
 
 static cudaError_t zero_state(f2_store* s, cudaStream_t st)
 {
-    cudaError_t e = cudaSuccess;
-    auto z = [&](void* p, size_t bytes) {
-        if (e == cudaSuccess && bytes) e = cudaMemsetAsync(p, 0, bytes, st);
-    };
-    z(s->rank, sizeof(int32_t) * (size_t)s->num_ctx);
-    z(s->contra, (size_t)s->num_ctx);
-    z(s->n_contra, sizeof(unsigned long long) * (size_t)s->num_ctx);
-    z(s->rows_seen, sizeof(long long) * (size_t)s->num_ctx);
-    z(s->pivot, sizeof(uint32_t) * (size_t)s->pivot_words);
-    z(s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
-    z(s->bz, sizeof(uint4) * (size_t)s->slots);
-    if (e == cudaSuccess && s->num_ctx)  // first_contra = -1 (all bytes 0xff)
-        e = cudaMemsetAsync(s->first_contra, 0xff, sizeof(long long) * (size_t)s->num_ctx, st);
-    z(s->status, sizeof(int));
-    return e;
+    F2FillList L;  // one launch for the whole state
+    L.add(s->rank, sizeof(int32_t) * (size_t)s->num_ctx);
+    L.add(s->contra, (size_t)s->num_ctx);
+    L.add(s->n_contra, sizeof(unsigned long long) * (size_t)s->num_ctx);
+    L.add(s->rows_seen, sizeof(long long) * (size_t)s->num_ctx);
+    L.add(s->pivot, sizeof(uint32_t) * (size_t)s->pivot_words);
+    L.add(s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
+    L.add(s->bz, sizeof(uint4) * (size_t)s->slots);
+    L.add(s->first_contra, sizeof(long long) * (size_t)s->num_ctx, 0xff);  // -1
+    L.add(s->status, sizeof(int));
+    return f2_fill(L, st);
 }
 
 extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_host, uint32_t flags,
@@ -122,6 +156,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->dedup = 1;
     s->elim_tables = 1;
     s->small_basis_bytes = DEFAULT_SMALL_REGION_BYTES;
+    s->dd_shards = 4;
     s->enc_table_min = f2_encode_table_min_default();
     s->enc_chunk_shift = f2_encode_chunk_shift_default();
     s->enc_chunk_min = f2_encode_chunk_min_default();
@@ -175,11 +210,14 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     alloc((void**)&s->bx, sizeof(uint32_t) * (size_t)s->basis_words);
     alloc((void**)&s->bz, sizeof(uint4) * (size_t)s->slots);
     alloc((void**)&s->status, sizeof(int));
-    alloc((void**)&s->queue, sizeof(int32_t) * C);
+    // the queue also holds the shard items of split contexts
+    alloc((void**)&s->queue, sizeof(int32_t) * (C + (size_t)f2_shard_queue_extra(s->num_sms)));
     alloc((void**)&s->keybuf, sizeof(int32_t) * C);
     alloc((void**)&s->counters, sizeof(int) * CNT_WORDS);
     alloc((void**)&s->rep_count, sizeof(int32_t) * C);
-    alloc((void**)&s->plan_hist, sizeof(int) * PLAN_HIST_WORDS);
+    alloc((void**)&s->shard_reps, sizeof(int32_t) * 8 * C);
+    alloc((void**)&s->shard_done, sizeof(int32_t) * C);
+    alloc((void**)&s->plan_hist, sizeof(int) * 2 * PLAN_HIST_WORDS);  // the two plans of a learn call
     alloc((void**)&s->full_ctr, sizeof(int) * (4 * C + 1));
     alloc((void**)&s->full_cnt, sizeof(unsigned long long) * C);
     alloc((void**)&s->full_first, sizeof(unsigned long long) * C);
@@ -452,6 +490,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_SMALL_BASIS_BYTES:
         if (value < 4096 || value > 24576) return F2_ERR_INVALID_ARG;
         s->small_basis_bytes = (value / 16) * 16;
+        return F2_OK;
+    case F2_OPT_DEDUP_SHARDS:
+        if (value < 1 || value > 8) return F2_ERR_INVALID_ARG;
+        s->dd_shards = (int)value;
         return F2_OK;
     case F2_OPT_TIMING:
         if (value != 0 && value != 1) return F2_ERR_INVALID_ARG;

@@ -165,6 +165,23 @@ def test_config2_scaled(env, mode):
     _check_store(binding, st, O, queries=(q.ctx_id, q.x))
 
 
+@pytest.mark.parametrize("shards", [1, 2, 3, 8])
+def test_dedup_shards(env, shards):
+    """Contexts far above their share of a call's rows have their duplicate
+    pass split over several CTAs (F2_OPT_DEDUP_SHARDS at most): a row equal
+    to one of an earlier shard is then classified by the elimination instead,
+    and every exported array, the solve and the encode stay the oracle's."""
+    binding, dev = env
+    wl = wlmod.generate(wlmod.scaled(2, 48, rows_median=3000, rows_max=40000, n_contra=6), 2024)
+    assert int(wl.rows.max()) > 16384  # split 8 ways: far above 1/(4 x SMs) of the rows
+    st = binding.Store(wl.n_bits, device=dev)
+    st.set_option(binding.F2_OPT_DEDUP_SHARDS, shards)
+    gpu_learn_workload(binding, st, wl, dev)
+    O = oracle_for(wl)
+    q = wlmod.make_queries(wl, dict(ctx_mode=1, count=20000, zipf_s=1.1, out_frac=0.05), 98)
+    _check_store(binding, st, O, queries=(q.ctx_id, q.x))
+
+
 def test_config3_scaled(env):
     binding, dev = env
     wl = wlmod.generate(wlmod.scaled(3, 1500), 303, query_count=50000)
