@@ -5,9 +5,13 @@
 // rows each; contexts are independent, so chunk-wise learning gives the same
 // state as one call).  A private copy stream moves chunk j + 1 into the other
 // half of a double buffer while the caller's stream learns chunk j; events
-// order each half's reuse.  Encode calls are cut into chunks of queries with a
-// third stage: the words of chunk j go back to the host on a second private
-// stream while chunk j + 1 is encoded and chunk j + 2 is copied in.  Host
+// order each half's reuse; the chunk whose largest context is smallest goes
+// last (what is left after the last copy is that chunk's learn, which its
+// largest context bounds).  Encode calls are cut into chunks of queries with
+// a third stage: the words of chunk j go back to the host on a second
+// private stream while chunk j + 1 is encoded; the queries go in through a
+// ring of ENC_IN buffers, so up to ENC_IN chunks are copied in ahead of the
+// encoding (and of whatever the caller's stream runs before it).  Host
 // arrays are read (and host outputs written) asynchronously: they must stay
 // valid until the caller's stream has passed the call.
 #include <algorithm>
@@ -19,10 +23,13 @@ using namespace f2;
 
 namespace f2 {
 
+constexpr int ENC_IN = 4;  // query input buffers of f2_encode_host
+
 struct HostIO {
     int device = -1;
     cudaStream_t h2d = nullptr, d2h = nullptr;
     cudaEvent_t copied[2] = {}, freed[2] = {}, done[2] = {}, drained[2] = {}, last = nullptr;
+    cudaEvent_t qcopied[ENC_IN] = {}, qused[ENC_IN] = {};
     // learn chunks: feature words, 128-bit words, CSR slices (double buffered);
     // the rebased offsets of the current chunk (one buffer: rebased and used
     // on the caller's stream in order)
@@ -34,9 +41,9 @@ struct HostIO {
     int64_t* row_off = nullptr;
     int64_t* x_off = nullptr;
     int64_t full_cap = 0;
-    // encode chunks
-    int32_t* qc[2] = {};
-    uint32_t* qx[2] = {};
+    // encode chunks: inputs in a ring, outputs double buffered
+    int32_t* qc[ENC_IN] = {};
+    uint32_t* qx[ENC_IN] = {};
     uint4* qy[2] = {};
     uint8_t* qs[2] = {};
     int64_t q_cap = 0, qx_cap = 0;
@@ -85,6 +92,10 @@ int host_io(f2_store* st, HostIO** out)
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->done[b], cudaEventDisableTiming);
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->drained[b], cudaEventDisableTiming);
         }
+        for (int b = 0; b < ENC_IN && e == cudaSuccess; ++b) {
+            e = cudaEventCreateWithFlags(&h->qcopied[b], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->qused[b], cudaEventDisableTiming);
+        }
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->last, cudaEventDisableTiming);
         st->hio = h;
         if (e != cudaSuccess) return f2_cuda_status(e);
@@ -109,6 +120,7 @@ cudaError_t grow(const f2_store* st, T*& p, int64_t& cap, int64_t need)
 struct Chunk {
     int32_t c0, c1;
     int64_t r0, r1, xa, xb;
+    int64_t max_rows;  // rows of its largest context
 };
 
 }  // namespace
@@ -120,12 +132,18 @@ void f2_host_io_free(f2_store* st)
     if (h->h2d) cudaStreamSynchronize(h->h2d);
     if (h->d2h) cudaStreamSynchronize(h->d2h);
     for (int b = 0; b < 2; ++b) {
-        void* bufs[] = {h->x[b], h->y[b], h->ro[b], h->xo[b], h->qc[b], h->qx[b], h->qy[b], h->qs[b]};
+        void* bufs[] = {h->x[b], h->y[b], h->ro[b], h->xo[b], h->qy[b], h->qs[b]};
         for (void* p : bufs)
             if (p) cudaFree(p);
         cudaEvent_t evs[] = {h->copied[b], h->freed[b], h->done[b], h->drained[b]};
         for (cudaEvent_t ev : evs)
             if (ev) cudaEventDestroy(ev);
+    }
+    for (int b = 0; b < ENC_IN; ++b) {
+        if (h->qc[b]) cudaFree(h->qc[b]);
+        if (h->qx[b]) cudaFree(h->qx[b]);
+        if (h->qcopied[b]) cudaEventDestroy(h->qcopied[b]);
+        if (h->qused[b]) cudaEventDestroy(h->qused[b]);
     }
     if (h->last) cudaEventDestroy(h->last);
     if (h->row_off) cudaFree(h->row_off);
@@ -147,7 +165,7 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
     // validate the CSR batch on the host and cut it into chunks
     const int64_t target = st->host_chunk_bytes;
     std::vector<Chunk> chunks;
-    Chunk cur{0, 0, row_off[0], row_off[0], INT64_MAX, 0};
+    Chunk cur{0, 0, row_off[0], row_off[0], INT64_MAX, 0, 0};
     int64_t bytes = 0;
     for (int32_t c = 0; c < C; ++c) {
         const int64_t a0 = row_off[c], a1 = row_off[c + 1], rows = a1 - a0;
@@ -158,6 +176,7 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
         if (rows > 0) {
             cur.xa = std::min(cur.xa, x_off[c]);
             cur.xb = std::max(cur.xb, x_off[c] + rows * xw);
+            cur.max_rows = std::max(cur.max_rows, rows);
         }
         cur.c1 = c + 1;
         cur.r1 = a1;
@@ -167,11 +186,15 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
                 if (cur.xa == INT64_MAX) cur.xa = cur.xb = 0;
                 chunks.push_back(cur);
             }
-            cur = Chunk{c + 1, c + 1, a1, a1, INT64_MAX, 0};
+            cur = Chunk{c + 1, c + 1, a1, a1, INT64_MAX, 0, 0};
             bytes = 0;
         }
     }
     if (chunks.empty()) return F2_OK;
+    // contexts are independent, so the chunks may go in any order: the one
+    // with the smallest largest context last
+    std::stable_sort(chunks.begin(), chunks.end(),
+                     [](const Chunk& a, const Chunk& b) { return a.max_rows > b.max_rows; });
     HostIO* h = nullptr;
     int rc = host_io(st, &h);
     if (rc != F2_OK) return rc;
@@ -266,12 +289,15 @@ extern "C" int f2_encode_host(const f2_store* cst, int64_t Q, const int32_t* ctx
     cudaError_t e = cudaSuccess;
     if (qn > h->q_cap || qn * x_stride_words > h->qx_cap) {
         e = sync_all(h, cs);
-        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
-            int64_t a = h->q_cap, a2 = h->q_cap, a3 = h->q_cap, ax = h->qx_cap;
+        for (int b = 0; b < ENC_IN && e == cudaSuccess; ++b) {
+            int64_t a = h->q_cap, ax = h->qx_cap;
             e = grow(st, h->qc[b], a, qn);
-            if (e == cudaSuccess) e = grow(st, h->qy[b], a2, qn);
-            if (e == cudaSuccess) e = grow(st, h->qs[b], a3, qn);
             if (e == cudaSuccess) e = grow(st, h->qx[b], ax, qn * x_stride_words);
+        }
+        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+            int64_t a2 = h->q_cap, a3 = h->q_cap;
+            e = grow(st, h->qy[b], a2, qn);
+            if (e == cudaSuccess) e = grow(st, h->qs[b], a3, qn);
         }
         if (e != cudaSuccess) {
             h->q_cap = h->qx_cap = 0;  // a buffer may have been freed: regrow every one next time
@@ -283,23 +309,24 @@ extern "C" int f2_encode_host(const f2_store* cst, int64_t Q, const int32_t* ctx
     int j = 0;
     for (int64_t q0 = 0; q0 < Q; q0 += qn, ++j) {
         const int64_t n = std::min(qn, Q - q0);
-        const int b = j & 1;
-        // in: the half's inputs are free once its encode two chunks back is done
-        e = cudaStreamWaitEvent(h->h2d, h->done[b], 0);
+        const int b = j & 1, bi = j % ENC_IN;
+        // in: the input buffer is free once the encode ENC_IN chunks back is done
+        e = cudaStreamWaitEvent(h->h2d, h->qused[bi], 0);
         if (e == cudaSuccess)
-            e = cudaMemcpyAsync(h->qc[b], ctx_id + q0, sizeof(int32_t) * (size_t)n, cudaMemcpyHostToDevice, h->h2d);
+            e = cudaMemcpyAsync(h->qc[bi], ctx_id + q0, sizeof(int32_t) * (size_t)n, cudaMemcpyHostToDevice, h->h2d);
         if (e == cudaSuccess)
-            e = cudaMemcpyAsync(h->qx[b], x + q0 * x_stride_words, sizeof(uint32_t) * (size_t)(n * x_stride_words),
+            e = cudaMemcpyAsync(h->qx[bi], x + q0 * x_stride_words, sizeof(uint32_t) * (size_t)(n * x_stride_words),
                                 cudaMemcpyHostToDevice, h->h2d);
-        if (e == cudaSuccess) e = cudaEventRecord(h->copied[b], h->h2d);
+        if (e == cudaSuccess) e = cudaEventRecord(h->qcopied[bi], h->h2d);
         // encode: needs the inputs, and the half's outputs read out
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, h->copied[b], 0);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, h->qcopied[bi], 0);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, h->drained[b], 0);
         if (e != cudaSuccess) return f2_cuda_status(e);
-        rc = f2_encode_batched(st, n, h->qc[b], h->qx[b], x_stride_words, reinterpret_cast<uint32_t*>(h->qy[b]),
+        rc = f2_encode_batched(st, n, h->qc[bi], h->qx[bi], x_stride_words, reinterpret_cast<uint32_t*>(h->qy[b]),
                                h->qs[b], stream);
         if (rc != F2_OK) return rc;
-        e = cudaEventRecord(h->done[b], cs);
+        e = cudaEventRecord(h->qused[bi], cs);
+        if (e == cudaSuccess) e = cudaEventRecord(h->done[b], cs);
         // out
         if (e == cudaSuccess) e = cudaStreamWaitEvent(h->d2h, h->done[b], 0);
         if (e == cudaSuccess)

@@ -1676,6 +1676,16 @@ inline bool is_aligned(const void* p, size_t al) { return ((uintptr_t)p % al) ==
 // the first contradicting row and rows_seen.
 // ---------------------------------------------------------------------------
 constexpr int FULL_STAGE = FULL_THREADS;  // rows staged in shared memory at a time (one per thread)
+// The table: low and high halves of the 16 entries of each group of four
+// coordinates in two planes of 8-byte entries (a warp's lookups at one group
+// fall in distinct banks), groups padded with zero entries to a multiple of
+// eight (one 32-bit word of q = eight lookups, no bounds test), the high
+// plane at a fixed distance from the low one and the base 1024-byte aligned,
+// so that an entry's address is the word's base OR the nibble times eight,
+// with the group and the plane in the loads' immediate offsets.
+constexpr int FULL_NP_MAX = 8 * ((MAX_D + 31) / 32);      // 264 groups
+constexpr int FULL_ZH_BYTES = FULL_NP_MAX * 16 * 8;        // 33,792: low plane, then the high plane
+constexpr int FULL_TABLE_WORDS = 2 * FULL_ZH_BYTES / 4 + 256;  // both planes + alignment slack
 
 struct FullArgs {
     const int64_t* row_off;
@@ -1690,14 +1700,16 @@ struct FullArgs {
     const int32_t* late_start;        // their first row left
     unsigned long long* cnt;          // [C] contradicting rows of the call
     unsigned long long* first;        // [C] first contradicting row of the call (all ones: none)
-    int table_words;                  // >= 64 * ceil(d / 4) for every context
+    int table_words;                  // FULL_TABLE_WORDS
 };
 
 __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, FullArgs a)
 {
     extern __shared__ uint4 full_smem[];
-    uint32_t* const tabw = reinterpret_cast<uint32_t*>(full_smem);
-    uint32_t* const stage = tabw + a.table_words;
+    // the table at the first 1024-byte boundary of the dynamic shared memory
+    const uint32_t pad = ((1024u - (smem_addr(full_smem) & 1023u)) & 1023u) / 4u;
+    uint32_t* const tabw = reinterpret_cast<uint32_t*>(full_smem) + pad;
+    uint32_t* const stage = reinterpret_cast<uint32_t*>(full_smem) + a.table_words;
     __shared__ int s_q, s_k;
     __shared__ unsigned long long s_cnt, s_first;
     const int t = threadIdx.x, lane = t & 31;
@@ -1730,8 +1742,9 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
         const int64_t i_first = start_of(q, c);
         const CtxDesc cd = s.desc[c];
         const int np = (cd.d + 3) >> 2;
+        const int nw = (np + 7) >> 3;  // words of q, eight groups each
         uint2* Zl = reinterpret_cast<uint2*>(tabw);
-        uint2* Zh = Zl + np * 16;
+        uint2* Zh = Zl + FULL_ZH_BYTES / 8;
         if (built != c) {
             for (int j = t; j < 4 * np; j += FULL_THREADS) {
                 const uint4 z = (j < cd.d) ? __ldg(s.bz + cd.slot_off + j) : make_uint4(0, 0, 0, 0);
@@ -1761,6 +1774,10 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
                 }
                 Zl[f] = lo;
                 Zh[f] = hi;
+            }
+            for (int f = 16 * np + t; f < 128 * nw; f += FULL_THREADS) {  // padding groups
+                Zl[f] = make_uint2(0, 0);
+                Zh[f] = make_uint2(0, 0);
             }
             built = c;
         }
@@ -1798,9 +1815,8 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
                 const uint4 yi = __ldg(a.y + r0 + i);
                 const uint32_t* xr = stage + t * sst;
                 uint32_t a0 = 0, a1 = 0, a2 = 0, a3 = 0, prev = 0;
-                const uint2* zl = Zl;
-                const uint2* zh = Zh;
-                for (int w = 0, left = np; left > 0; ++w, left -= 8, zl += 128, zh += 128) {
+                const char* const zt = reinterpret_cast<const char*>(tabw);
+                for (int w = 0; w < nw; ++w) {
                     uint32_t xv = (w < xw) ? xr[w] : 0u;
                     if (w == xw - 1) xv &= lm;
                     uint32_t qw;
@@ -1810,16 +1826,20 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
                         qw = (xv << 1) | (prev >> 31) | (w == 0 ? 1u : 0u);
                         prev = xv;
                     }
+                    const char* const zb = zt + w * 1024;
+                    // two lookups a step: entry byte offset = nibble * 8
 #pragma unroll
-                    for (int h = 0; h < 8; ++h) {
-                        if (h < left) {
-                            const int e = h * 16 + (int)((qw >> (4 * h)) & 15u);
-                            const uint2 lo = zl[e], hi = zh[e];
-                            a0 ^= lo.x;
-                            a1 ^= lo.y;
-                            a2 ^= hi.x;
-                            a3 ^= hi.y;
-                        }
+                    for (int h = 0; h < 8; h += 2) {
+                        const uint32_t oa = (h == 0) ? ((qw << 3) & 0x78u) : ((qw >> (4 * h - 3)) & 0x78u);
+                        const uint32_t ob = (qw >> (4 * h + 1)) & 0x78u;
+                        const uint2 la = *reinterpret_cast<const uint2*>(zb + oa + 128 * h);
+                        const uint2 ha = *reinterpret_cast<const uint2*>(zb + oa + FULL_ZH_BYTES + 128 * h);
+                        const uint2 lb = *reinterpret_cast<const uint2*>(zb + ob + 128 * (h + 1));
+                        const uint2 hb = *reinterpret_cast<const uint2*>(zb + ob + FULL_ZH_BYTES + 128 * (h + 1));
+                        a0 ^= la.x ^ lb.x;
+                        a1 ^= la.y ^ lb.y;
+                        a2 ^= ha.x ^ hb.x;
+                        a3 ^= ha.y ^ hb.y;
                     }
                 }
                 if (a0 != yi.x || a1 != yi.y || a2 != yi.z || a3 != yi.w) {
@@ -2016,7 +2036,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
         fa.late_start = lx.late_start;
         fa.cnt = full_cnt;
         fa.first = full_first;
-        fa.table_words = 64 * ((wv.max_d + 3) / 4);
+        fa.table_words = FULL_TABLE_WORDS;
         const size_t smem = 4 * ((size_t)fa.table_words + (size_t)FULL_STAGE * (size_t)(wv.max_xw | 1));
         e = cudaFuncSetAttribute(verify_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return f2_cuda_status(e);
