@@ -151,18 +151,54 @@ template <int RW, int WD>
 __device__ __forceinline__ void table_reduce(const uint32_t* tab, int np, uint32_t (&q)[WD], uint4& acc,
                                              uint32_t (&r)[RW > 0 ? RW : 1])
 {
-    const uint2* Zl = reinterpret_cast<const uint2*>(tab);
-    const uint2* Zh = Zl + np * 16;
-    const uint32_t* R = tab + 64 * np;
-    const int rstride = 16 * np;
+    // byte addressing: entry v of group h of a word sits at 8v (16v in the
+    // residual planes: 4v) bytes from the word's plane bases, with the
+    // group's offset an immediate; two lookups per step share three-input XORs
+    const char* const base = reinterpret_cast<const char*>(tab);
+    const int zh_off = np * 128;       // high plane, bytes from the low one
+    const int r_off = np * 256;        // first residual plane
+    const int r_stride = np * 64;      // between residual planes
     uint32_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
 #pragma unroll
     for (int u = 0; u < (RW > 0 ? RW : 1); ++u) r[u] = 0;
+    int left = np;
+    int wo = 0;  // the word's byte offset in the low plane (1024 a word; 512 in a residual plane)
 #pragma unroll 1
-    for (int left = np; left > 0; left -= 8) {
+    for (; left >= 8; left -= 8, wo += 1024) {  // whole words of eight groups: no bounds test
         const uint32_t word = q[0];
 #pragma unroll
         for (int v = 0; v < WD - 1; ++v) q[v] = q[v + 1];
+        const char* const zl = base + wo;
+        const char* const zh = zl + zh_off;
+        const char* const rp = base + r_off + (wo >> 1);
+#pragma unroll
+        for (int h = 0; h < 8; h += 2) {
+            const uint32_t oa = (h == 0) ? ((word << 3) & 0x78u) : ((word >> (4 * h - 3)) & 0x78u);
+            const uint32_t ob = (word >> (4 * h + 1)) & 0x78u;
+            const uint2 la = *reinterpret_cast<const uint2*>(zl + oa + 128 * h);
+            const uint2 lb = *reinterpret_cast<const uint2*>(zl + ob + 128 * (h + 1));
+            const uint2 ha = *reinterpret_cast<const uint2*>(zh + oa + 128 * h);
+            const uint2 hb = *reinterpret_cast<const uint2*>(zh + ob + 128 * (h + 1));
+            a0 ^= la.x ^ lb.x;
+            a1 ^= la.y ^ lb.y;
+            a2 ^= ha.x ^ hb.x;
+            a3 ^= ha.y ^ hb.y;
+#pragma unroll
+            for (int u = 0; u < RW; ++u) {
+                const char* ru = rp + u * r_stride;
+                r[u] ^= *reinterpret_cast<const uint32_t*>(ru + (oa >> 1) + 64 * h) ^
+                        *reinterpret_cast<const uint32_t*>(ru + (ob >> 1) + 64 * (h + 1));
+            }
+        }
+    }
+    if (left > 0) {  // the last word's groups
+        const uint32_t word = q[0];
+#pragma unroll
+        for (int v = 0; v < WD - 1; ++v) q[v] = q[v + 1];
+        const int g0 = np - left;  // its first group
+        const uint2* Zl = reinterpret_cast<const uint2*>(tab) + 16 * g0;
+        const uint2* Zh = Zl + np * 16;
+        const uint32_t* R = tab + 64 * np + 16 * g0;
 #pragma unroll
         for (int h = 0; h < 8; ++h) {
             if (h < left) {
@@ -174,12 +210,9 @@ __device__ __forceinline__ void table_reduce(const uint32_t* tab, int np, uint32
                 a2 ^= hi.x;
                 a3 ^= hi.y;
 #pragma unroll
-                for (int u = 0; u < RW; ++u) r[u] ^= R[u * rstride + e];
+                for (int u = 0; u < RW; ++u) r[u] ^= R[u * (16 * np) + e];
             }
         }
-        Zl += 128;
-        Zh += 128;
-        R += 128;
     }
     acc = make_uint4(a0, a1, a2, a3);
 }

@@ -3,9 +3,10 @@
 //
 // A learn call is cut into chunks of whole contexts (about chunk_bytes of
 // rows each; contexts are independent, so chunk-wise learning gives the same
-// state as one call).  A private copy stream moves chunk j + 1 into the other
-// half of a double buffer while the caller's stream learns chunk j; events
-// order each half's reuse; the chunk whose largest context is smallest goes
+// state as one call).  A private copy stream moves chunks into a ring of
+// LEARN_BUFS buffers while the caller's stream learns the ones before;
+// events order each buffer's reuse; the chunk whose largest context is
+// smallest goes
 // last (what is left after the last copy is that chunk's learn, which its
 // largest context bounds).  Encode calls are cut into chunks of queries with
 // a third stage: the words of chunk j go back to the host on a second
@@ -23,20 +24,21 @@ using namespace f2;
 
 namespace f2 {
 
-constexpr int ENC_IN = 4;  // query input buffers of f2_encode_host
+constexpr int ENC_IN = 4;      // query input buffers of f2_encode_host
+constexpr int LEARN_BUFS = 2;  // chunk buffers of f2_learn_host (four measured no faster)
 
 struct HostIO {
     int device = -1;
     cudaStream_t h2d = nullptr, d2h = nullptr;
-    cudaEvent_t copied[2] = {}, freed[2] = {}, done[2] = {}, drained[2] = {}, last = nullptr;
+    cudaEvent_t copied[LEARN_BUFS] = {}, freed[LEARN_BUFS] = {}, done[2] = {}, drained[2] = {}, last = nullptr;
     cudaEvent_t qcopied[ENC_IN] = {}, qused[ENC_IN] = {};
-    // learn chunks: feature words, 128-bit words, CSR slices (double buffered);
-    // the rebased offsets of the current chunk (one buffer: rebased and used
-    // on the caller's stream in order)
-    uint32_t* x[2] = {};
-    uint4* y[2] = {};
-    int64_t* ro[2] = {};
-    int64_t* xo[2] = {};
+    // learn chunks: feature words, 128-bit words, CSR slices (a ring); the
+    // rebased offsets of the current chunk (one buffer: rebased and used on
+    // the caller's stream in order)
+    uint32_t* x[LEARN_BUFS] = {};
+    uint4* y[LEARN_BUFS] = {};
+    int64_t* ro[LEARN_BUFS] = {};
+    int64_t* xo[LEARN_BUFS] = {};
     int64_t x_cap = 0, y_cap = 0, c_cap = 0;
     int64_t* row_off = nullptr;
     int64_t* x_off = nullptr;
@@ -86,10 +88,12 @@ int host_io(f2_store* st, HostIO** out)
         cudaError_t e = cudaGetDevice(&h->device);
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->h2d, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking);
-        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+        for (int b = 0; b < LEARN_BUFS && e == cudaSuccess; ++b) {
             e = cudaEventCreateWithFlags(&h->copied[b], cudaEventDisableTiming);
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->freed[b], cudaEventDisableTiming);
-            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->done[b], cudaEventDisableTiming);
+        }
+        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+            e = cudaEventCreateWithFlags(&h->done[b], cudaEventDisableTiming);
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->drained[b], cudaEventDisableTiming);
         }
         for (int b = 0; b < ENC_IN && e == cudaSuccess; ++b) {
@@ -131,11 +135,19 @@ void f2_host_io_free(f2_store* st)
     if (!h) return;
     if (h->h2d) cudaStreamSynchronize(h->h2d);
     if (h->d2h) cudaStreamSynchronize(h->d2h);
-    for (int b = 0; b < 2; ++b) {
-        void* bufs[] = {h->x[b], h->y[b], h->ro[b], h->xo[b], h->qy[b], h->qs[b]};
+    for (int b = 0; b < LEARN_BUFS; ++b) {
+        void* bufs[] = {h->x[b], h->y[b], h->ro[b], h->xo[b]};
         for (void* p : bufs)
             if (p) cudaFree(p);
-        cudaEvent_t evs[] = {h->copied[b], h->freed[b], h->done[b], h->drained[b]};
+        cudaEvent_t evs[] = {h->copied[b], h->freed[b]};
+        for (cudaEvent_t ev : evs)
+            if (ev) cudaEventDestroy(ev);
+    }
+    for (int b = 0; b < 2; ++b) {
+        void* bufs[] = {h->qy[b], h->qs[b]};
+        for (void* p : bufs)
+            if (p) cudaFree(p);
+        cudaEvent_t evs[] = {h->done[b], h->drained[b]};
         for (cudaEvent_t ev : evs)
             if (ev) cudaEventDestroy(ev);
     }
@@ -208,7 +220,7 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
     cudaError_t e = cudaSuccess;
     if (need_x > h->x_cap || need_y > h->y_cap || need_c > h->c_cap || C + 1 > h->full_cap) {
         e = sync_all(h, cs);
-        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+        for (int b = 0; b < LEARN_BUFS && e == cudaSuccess; ++b) {
             int64_t xc = h->x_cap, yc = h->y_cap, cc = h->c_cap, cc2 = h->c_cap;
             e = grow(st, h->x[b], xc, need_x);
             if (e == cudaSuccess) e = grow(st, h->y[b], yc, need_y);
@@ -232,9 +244,9 @@ extern "C" int f2_learn_host(f2_store* st, const int64_t* row_off, const uint32_
     }
     for (size_t j = 0; j < chunks.size(); ++j) {
         const Chunk& k = chunks[j];
-        const int b = (int)(j & 1);
+        const int b = (int)(j % LEARN_BUFS);
         const int64_t nc = k.c1 - k.c0;
-        // copy stream: this half is free once the learn two chunks back is done
+        // copy stream: this buffer is free once the learn LEARN_BUFS chunks back is done
         e = cudaStreamWaitEvent(h->h2d, h->freed[b], 0);
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(h->ro[b], row_off + k.c0, sizeof(int64_t) * (size_t)(nc + 1),
