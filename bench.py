@@ -740,14 +740,16 @@ def launches_per_step(wl, has_q: bool) -> int:
     the elimination kernel of each width class present (d <= 96, 96 < d <=
     288, 288 < d <= 544, wider) and the full-rank check; solve_kernel; per
     2^25 queries the encode's fill and its seven kernels (count, table,
-    build, scan, scatter, runs, short)."""
+    build, scan, scatter, runs, short), or one kernel for a pass of at most
+    65,536 queries."""
     wd = (wl.n_bits.astype(np.int64) + 1 + 31) // 32
     xw = (wl.n_bits.astype(np.int64) + 31) // 32
     plan = 1 if wl.num_ctx <= 8192 else 3
     elim = (int((wd <= 3).any()) + int(((wd > 3) & (wd <= 9)).any()) + int(((wd > 9) & (wd <= 17)).any())
             + int((wd > 17).any()))
     learn = 1 + plan + 1 + int((xw > 9).any()) + plan + elim + 1
-    enc = 8 * ((len(wl.queries.ctx_id) + (1 << 25) - 1) >> 25) if has_q else 0
+    nq = len(wl.queries.ctx_id) if has_q else 0
+    enc = (1 if nq <= 65536 else 8 * ((nq + (1 << 25) - 1) >> 25)) if has_q else 0
     return 1 + len(wl.batches) * learn + 1 + enc
 
 

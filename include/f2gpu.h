@@ -317,6 +317,9 @@ enum f2_option {
                                     of the call's rows x (feature words + 4) the context holds, and
                                     at least one per 16384 rows); default 4, in [1, 8]; 1 = never
                                     split (and no 4-warp context promoted to a whole CTA) */
+    F2_OPT_ENCODE_DIRECT_MAX = 14, /* f2_encode_batched calls of at most this many queries encode each
+                                    query on its own from the stored basis, with no grouping and no
+                                    tables (one kernel launch); default 65536, 0 = never */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -638,7 +638,7 @@ __device__ __forceinline__ void encode_direct(const StoreDev& s, int32_t c, int6
 {
     uint4 acc = make_uint4(0, 0, 0, 0);
     uint8_t flag;
-    if (c >= s.num_ctx) {
+    if ((uint32_t)c >= (uint32_t)s.num_ctx) {
         record_status(s.status, F2_ERR_CTX_RANGE);
         flag = 0xFF;
     } else {
@@ -1176,6 +1176,17 @@ __global__ void __launch_bounds__(SHORT_THREADS) enc_short_kernel(StoreDev s,
     }
 }
 
+// A small pass: every query on its own, its basis rows read from the store
+// (L2), no grouping -- one launch where the grouped path takes eight, which
+// is what a small batch waits for.
+__global__ void __launch_bounds__(256) enc_direct_kernel(StoreDev s, int32_t n, const int32_t* __restrict__ ctx_id,
+                                                         const uint32_t* __restrict__ x, int stride,
+                                                         uint4* __restrict__ y, uint8_t* __restrict__ in_span)
+{
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+        encode_direct(s, __ldg(ctx_id + i), i, x, stride, y, in_span);
+}
+
 }  // namespace
 
 extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* ctx_id, const uint32_t* x,
@@ -1188,6 +1199,13 @@ extern "C" int f2_encode_batched(const f2_store* st, int64_t Q, const int32_t* c
     if (((uintptr_t)y_out % 16) != 0 || ((uintptr_t)x % 4) != 0 || ((uintptr_t)ctx_id % 4) != 0)
         return F2_ERR_ALIGN;
     cudaStream_t cs = (cudaStream_t)stream;
+    if (Q <= st->enc_direct_max) {  // a small pass: no grouping, no scratch
+        int blocks = (int)((Q + 255) / 256);
+        if (blocks > 8 * st->num_sms) blocks = 8 * st->num_sms;
+        enc_direct_kernel<<<blocks, 256, 0, cs>>>(st->dev(), (int32_t)Q, ctx_id, x, x_stride_words,
+                                                 reinterpret_cast<uint4*>(y_out), in_span);
+        return f2_cuda_status(cudaGetLastError());
+    }
     const int64_t sub = Q < ENC_SUB ? Q : ENC_SUB;
     int shift = st->enc_chunk_shift;
     while ((sub >> shift) >= ENC_MAX_CHUNKS) ++shift;

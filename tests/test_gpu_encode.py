@@ -1,7 +1,8 @@
 """Encode paths (Sec. 2.3) vs the CPU oracle: queries grouped by context,
 long runs encoded with per-run lookup tables of the basis, the others by the
-per-query pivot walk.  Every run length, width and residual size that
-switches between the two is covered, with both paths forced on and off."""
+per-query pivot walk, and small passes with no grouping at all.  Every run
+length, width and residual size that switches between the paths is covered,
+with each path forced on and off."""
 import numpy as np
 import pytest
 import torch
@@ -14,6 +15,7 @@ from gpu_util import csr_from_rows, cuda_device, dev_arrays, gpu_learn_workload,
 pytestmark = pytest.mark.gpu
 
 TABLE_MINS = (16, 32, 200, 1 << 30)  # 1 << 30: tables off
+DIRECT = "direct"  # every query on its own (F2_OPT_ENCODE_DIRECT_MAX above the pass)
 
 
 @pytest.fixture(scope="module")
@@ -23,7 +25,11 @@ def env():
 
 
 def _encode_all(binding, st, ctx, qx, table_min):
-    st.set_option(binding.F2_OPT_ENCODE_TABLE_MIN, table_min)
+    if table_min == DIRECT:
+        st.set_option(binding.F2_OPT_ENCODE_DIRECT_MAX, 1 << 30)
+    else:  # the grouped path, whatever the pass size
+        st.set_option(binding.F2_OPT_ENCODE_DIRECT_MAX, 0)
+        st.set_option(binding.F2_OPT_ENCODE_TABLE_MIN, table_min)
     ct, xt = dev_arrays(binding, st.device, ctx, qx)
     y, ok = st.encode(ct, xt)
     torch.cuda.synchronize()
@@ -32,7 +38,7 @@ def _encode_all(binding, st, ctx, qx, table_min):
 
 def _compare(binding, st, O, ctx, qx, expect_status=0):
     ry, rok = O.encode(ctx, qx)
-    for tm in TABLE_MINS:
+    for tm in TABLE_MINS + (DIRECT,):
         y, ok = _encode_all(binding, st, ctx, qx, tm)
         bad = np.flatnonzero((ok != rok) | (y != ry).any(axis=1))
         assert bad.size == 0, (tm, bad[:8].tolist(), ctx[bad[:8]].tolist())
@@ -158,7 +164,7 @@ def test_bad_ids_and_stride_in_long_runs(env):
     assert (ok[ctx >= wl.num_ctx] == 0xFF).all() and (ok[ctx < 0] == 0xFF).all()
     wide = np.flatnonzero(wl.n_bits > 64).astype(np.int32)
     ctx2 = np.repeat(wide[:2], 100)
-    for tm in TABLE_MINS:
+    for tm in TABLE_MINS + (DIRECT,):
         yy, ok2 = _encode_all(binding, st, ctx2, qx[:200], tm)
         assert (ok2 == 0xFF).all() and not yy.any()
         assert st.device_status() == 9

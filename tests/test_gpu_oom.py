@@ -91,6 +91,7 @@ def test_oom_encode(env):
 
     def make():
         st = binding.Store(wl.n_bits, device=dev)
+        st.set_option(binding.F2_OPT_ENCODE_DIRECT_MAX, 0)  # the grouped path and its scratch
         gpu_learn_workload(binding, st, wl, dev)
         return st
 
