@@ -654,7 +654,7 @@ def run_ours(args):
     # learn roofline is HBM.  ops_learn is kept as the naive-method reference.
     learn_bound = "hbm"
     rl_learn = {
-        "kernel": "f2_learn_batched (plan kernels, dedup_kernel, elim_narrow_kernel<true/false>, "
+        "kernel": "f2_learn_batched (fill, plan kernels, dedup_kernel, elim_narrow_kernel<true/false>, "
                   "elim_wide_kernel, verify_full_kernel)",
         "hbm": {"achieved": bytes_learn / learn_mean / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": (bytes_learn / learn_mean) / hbm_peak, "bytes_per_launch": bytes_learn},
@@ -700,7 +700,8 @@ def run_ours(args):
         result["encode_words_per_s"] = Q / enc_mean
         result["encode_in_span_frac"] = float((span_np == 1).mean())
         result["roofline_encode"] = {
-            "kernel": "f2_encode_batched (enc_count, enc_scan, enc_scatter, enc_runs, enc_short kernels)",
+            "kernel": ("f2_encode_batched (fill, enc_count, enc_table, enc_build, enc_scan, enc_scatter, "
+                       "enc_runs, enc_short kernels; enc_direct alone for a pass of at most 65,536 queries)"),
             "hbm": {"achieved": bytes_enc / enc_mean / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                     "frac": bytes_enc / enc_mean / hbm_peak, "bytes_per_launch": bytes_enc},
             # per query the naive pivot walk's word XORs (|q AND P| x (wd + 4)):
