@@ -320,6 +320,9 @@ enum f2_option {
     F2_OPT_ENCODE_DIRECT_MAX = 14, /* f2_encode_batched calls of at most this many queries encode each
                                     query on its own from the stored basis, with no grouping and no
                                     tables (one kernel launch); default 65536, 0 = never */
+    F2_OPT_LONG_CALL_ROWS = 15,  /* f2_learn_batched calls of at least this many rows eliminate the contexts
+                                    of 4..9 words in CTAs of four warps instead of eight (more contexts
+                                    side by side; the longest contexts take longer); default 2^25 */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

@@ -42,6 +42,7 @@ F2_OPT_ELIM_TABLES = 11
 F2_OPT_SMALL_BASIS_BYTES = 12
 F2_OPT_DEDUP_SHARDS = 13
 F2_OPT_ENCODE_DIRECT_MAX = 14
+F2_OPT_LONG_CALL_ROWS = 15
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

@@ -33,6 +33,7 @@ constexpr int PLAN_BUCKETS = 48;     // log2(work) buckets for longest-first ord
 constexpr int DEFAULT_WARP_REGION_BYTES = 12288;  // shared memory of one warp-owned context
 constexpr int DEFAULT_SMALL_REGION_BYTES = 4096;  // the same in the small-width kernel (d <= 96)
 constexpr int64_t DEFAULT_ENCODE_DIRECT_MAX = 65536;  // encode passes this small skip the grouping
+constexpr int64_t DEFAULT_LONG_CALL_ROWS = int64_t(1) << 25;  // learn calls this long: 4-warp CTAs (4..9 words)
 constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA (at most)
 constexpr int HEAVY_ROWS_MIN = 1024;              // ... and at least, when it scales with the batch:
 constexpr int HEAVY_ROWS_BATCH_DIV = 20000;       // batch rows / this (no duplicate pass), or
@@ -353,6 +354,7 @@ struct f2_store {
     int64_t small_basis_bytes;  // shared memory of a warp-owned context, small-width kernel
     int dd_shards;              // most CTAs one context's duplicate pass is split over
     int64_t enc_direct_max;     // encode passes of at most this many queries skip the grouping
+    int64_t long_call_rows;     // learn calls of at least this many rows: 4-warp CTAs for 4..9-word contexts
     f2::Widths widths;      // width classes of the contexts (computed on first use)
     // second stream of the learn launches (kernels of independent width
     // classes run side by side), its fork and join events; created on first use

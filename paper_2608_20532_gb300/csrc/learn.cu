@@ -1314,8 +1314,14 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
 static_assert(DEFAULT_SMALL_REGION_BYTES / 4 >= 32 * SMALL_WD * row_stride(SMALL_WD) + CTL_WORDS + FL_WORDS,
               "a warp region holds the basis of any small-width context");
 
-template <bool SMALL>
-__global__ void __launch_bounds__(LEARN_WARPS * 32, SMALL ? 4 : 2) elim_narrow_kernel(StoreDev s, LearnArgs a)
+//
+// NW: warps of a CTA.  The 4..9-word kernel has an instance of four-warp CTAs
+// (four per SM, the same warps per SM) for long calls: a CTA-owned context's
+// insertions run one warp at a time while the group's other warps wait, so
+// smaller groups waste less; in a short call the longest CTA-owned contexts
+// bound the call and keep eight warps each.
+template <bool SMALL, int NW = LEARN_WARPS>
+__global__ void __launch_bounds__(NW * 32, SMALL ? 4 : 16 / NW) elim_narrow_kernel(StoreDev s, LearnArgs a)
 {
     constexpr int C_CTA = SMALL ? CLS_CTA_S : CLS_CTA;
     constexpr int C_WARP = SMALL ? CLS_WARP_S : CLS_WARP;
@@ -1885,12 +1891,16 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
 
 // Which elimination kernels a store needs, and their widest bases.
 
-size_t narrow_smem(int max_narrow_words, int warp_region_words)
+size_t narrow_smem(int max_narrow_words, int warp_region_words, int nw)
 {
     const size_t cta = 4 * (size_t)max_narrow_words;
-    const size_t warps = 4 * (size_t)LEARN_WARPS * (size_t)warp_region_words;
+    const size_t warps = 4 * (size_t)nw * (size_t)warp_region_words;
     return cta > warps ? cta : warps;
 }
+
+// Calls of at least this many rows run the 4..9-word elimination in CTAs of
+// four warps (see elim_narrow_kernel; F2_OPT_LONG_CALL_ROWS).
+constexpr int64_t LONG_CALL_ROWS = DEFAULT_LONG_CALL_ROWS;
 
 // A second stream for kernels that work on disjoint contexts: the first
 // such kernel goes to `aux` (forked from the caller's stream), the others to
@@ -1925,7 +1935,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
                        unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr, int scale = 0,
-                       bool prezeroed = false)
+                       bool prezeroed = false, int64_t long_rows = LONG_CALL_ROWS)
 {
     // prezeroed: the caller has cleared full_ctr's first 2C words and late
     // count, full_cnt, full_first (to -1) and hist
@@ -1965,16 +1975,16 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     int rc = launch_plan(sd, pa, num_sms, cs);
     if (rc != F2_OK) return rc;
     cudaError_t e;
-    auto narrow = [&](auto kernel, size_t smem, cudaStream_t ks) -> int {
+    auto narrow = [&](auto kernel, size_t smem, cudaStream_t ks, int nw) -> int {
         cudaError_t er = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         int per_sm = 0;
-        er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, LEARN_WARPS * 32, smem);
+        er = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, nw * 32, smem);
         if (er != cudaSuccess) return f2_cuda_status(er);
         if (per_sm < 1) per_sm = 1;
         LearnArgs lk = lx;
         lk.cta_region_words = (int)(smem / 4);
-        kernel<<<num_sms * per_sm, LEARN_WARPS * 32, smem, ks>>>(sd, lk);
+        kernel<<<num_sms * per_sm, nw * 32, smem, ks>>>(sd, lk);
         return f2_cuda_status(cudaGetLastError());
     };
     // the three width classes hold disjoint contexts: with a second stream
@@ -2010,13 +2020,17 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     if (wv.has_narrow) {
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
-        rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words), ks);
+        if (total_rows >= long_rows)
+            rc = narrow(elim_narrow_kernel<false, 4>, narrow_smem(wv.max_narrow_words, la.warp_region_words, 4), ks, 4);
+        else
+            rc = narrow(elim_narrow_kernel<false>, narrow_smem(wv.max_narrow_words, la.warp_region_words, LEARN_WARPS),
+                        ks, LEARN_WARPS);
         if (rc != F2_OK) return rc;
     }
     if (wv.has_small) {
         const cudaStream_t ks = f.next(left--);
         if (f.e != cudaSuccess) return f2_cuda_status(f.e);
-        rc = narrow(elim_narrow_kernel<true>, small_smem, ks);
+        rc = narrow(elim_narrow_kernel<true>, small_smem, ks, LEARN_WARPS);
         if (rc != F2_OK) return rc;
     }
     e = f.join();
@@ -2219,7 +2233,8 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     const int scale = dedup && !st->heavy_rows_set && !st->warp_work_set;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               heavy, st->warp_work, st->queue, st->keybuf, st->plan_hist + PLAN_HIST_WORDS,
-                              st->num_sms, wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale, true);
+                              st->num_sms, wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale, true,
+                              st->long_call_rows);
 }
 
 extern "C" int f2_learn_timing(const f2_store* st, uint64_t* out_host, f2_stream_t stream)
@@ -2362,6 +2377,7 @@ cudaError_t noalloc_load_kernels()
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_scatter_kernel);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<true>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<false>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<false, 4>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_wide_kernel<WIDE_WD, CLS_WIDE>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_wide_kernel<WIDE_M_WD, CLS_WIDE_M>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, verify_full_kernel);

@@ -158,6 +158,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->small_basis_bytes = DEFAULT_SMALL_REGION_BYTES;
     s->dd_shards = 4;
     s->enc_direct_max = DEFAULT_ENCODE_DIRECT_MAX;
+    s->long_call_rows = DEFAULT_LONG_CALL_ROWS;
     s->enc_table_min = f2_encode_table_min_default();
     s->enc_chunk_shift = f2_encode_chunk_shift_default();
     s->enc_chunk_min = f2_encode_chunk_min_default();
@@ -491,6 +492,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_SMALL_BASIS_BYTES:
         if (value < 4096 || value > 24576) return F2_ERR_INVALID_ARG;
         s->small_basis_bytes = (value / 16) * 16;
+        return F2_OK;
+    case F2_OPT_LONG_CALL_ROWS:
+        if (value < 0) return F2_ERR_INVALID_ARG;
+        s->long_call_rows = value;
         return F2_OK;
     case F2_OPT_ENCODE_DIRECT_MAX:
         if (value < 0 || value > (int64_t(1) << 30)) return F2_ERR_INVALID_ARG;

@@ -148,12 +148,14 @@ def test_config1(env):
     assert np.array_equal(np.flatnonzero(ex["contra"]), np.flatnonzero(wl.contra_pos >= 0))
 
 
-@pytest.mark.parametrize("mode", ["default", "all_cta", "all_warp"])
+@pytest.mark.parametrize("mode", ["default", "all_cta", "all_warp", "cta4", "all_cta4"])
 def test_config2_scaled(env, mode):
     binding, dev = env
     wl = wlmod.generate(wlmod.scaled(2, 400), 202)
     st = binding.Store(wl.n_bits, device=dev)
-    if mode == "all_cta":
+    if mode in ("cta4", "all_cta4"):  # the 4..9-word contexts' CTAs of four warps
+        st.set_option(binding.F2_OPT_LONG_CALL_ROWS, 0)
+    if mode in ("all_cta", "all_cta4"):
         st.set_option(binding.F2_OPT_HEAVY_ROWS, 1)
     if mode == "all_warp":
         st.set_option(binding.F2_OPT_HEAVY_ROWS, 1 << 40)
