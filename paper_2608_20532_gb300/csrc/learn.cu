@@ -1309,7 +1309,9 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
 
 // Narrow elimination: CTA-owned contexts first (longest first), then
 // warp-owned ones.  SMALL: the contexts of at most SMALL_WD words, with
-// fixed 4 KB warp regions and a register budget for four CTAs per SM; else
+// fixed 4 KB warp regions and a register budget for three CTAs per SM (80
+// registers, no spills; four CTAs at 64 registers spill and ran 6% slower
+// on the 78k-context, 81M-row learn); else
 // the contexts of SMALL_WD + 1 .. NARROW_WD words.
 static_assert(DEFAULT_SMALL_REGION_BYTES / 4 >= 32 * SMALL_WD * row_stride(SMALL_WD) + CTL_WORDS + FL_WORDS,
               "a warp region holds the basis of any small-width context");
@@ -1321,7 +1323,7 @@ static_assert(DEFAULT_SMALL_REGION_BYTES / 4 >= 32 * SMALL_WD * row_stride(SMALL
 // smaller groups waste less; in a short call the longest CTA-owned contexts
 // bound the call and keep eight warps each.
 template <bool SMALL, int NW = LEARN_WARPS>
-__global__ void __launch_bounds__(NW * 32, SMALL ? 4 : 16 / NW) elim_narrow_kernel(StoreDev s, LearnArgs a)
+__global__ void __launch_bounds__(NW * 32, SMALL ? 3 : 16 / NW) elim_narrow_kernel(StoreDev s, LearnArgs a)
 {
     constexpr int C_CTA = SMALL ? CLS_CTA_S : CLS_CTA;
     constexpr int C_WARP = SMALL ? CLS_WARP_S : CLS_WARP;
