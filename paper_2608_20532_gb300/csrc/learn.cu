@@ -1619,9 +1619,23 @@ __device__ __forceinline__ void plan_place(const PlanArgs& p, int* cursor, int c
 
 __global__ void __launch_bounds__(256) plan_scatter_kernel(StoreDev s, PlanArgs p)
 {
-    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < s.num_ctx; c += gridDim.x * blockDim.x) {
-        const int kv = p.keybuf[c];
-        if (kv >= 0) plan_place(p, p.hist, c, kv);
+    // the lanes of a warp with the same key take their slots with one atomic
+    const int lane = threadIdx.x & 31;
+    for (int b = blockIdx.x * blockDim.x; b < s.num_ctx; b += gridDim.x * blockDim.x) {
+        const int c = b + (int)threadIdx.x;
+        const int kv = (c < s.num_ctx) ? p.keybuf[c] : -1;
+        const bool single = kv >= 0 && (kv >> 16) == 0;
+        const int key = single ? kv : -1 - lane;  // a lane of its own unless a single item
+        const unsigned peers = __match_any_sync(FULL, key);
+        if (single) {
+            const int leader = __ffs(peers) - 1;
+            int q0 = 0;
+            if (lane == leader) q0 = atomicAdd(p.hist + key, __popc(peers));
+            q0 = __shfl_sync(peers, q0, leader);
+            p.queue[q0 + __popc(peers & ((1u << lane) - 1u))] = c;
+        } else if (kv >= 0) {
+            plan_place(p, p.hist, c, kv);
+        }
     }
 }
 
@@ -2377,6 +2391,7 @@ cudaError_t noalloc_load_kernels()
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_key_kernel);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_scan_kernel);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_scatter_kernel);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, plan_small_kernel);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<true>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<false>);
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, elim_narrow_kernel<false, 4>);
