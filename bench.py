@@ -683,8 +683,8 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "u32", "data": "synthetic (seeded planted affine maps)",
-        "config": dict(describe(cfg_id, wl), parallelism=f"replicas x{world}" if world > 1 else "single GPU",
-                       launch=launch_mode),
+        "config": dict(describe(cfg_id, wl), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
+        "launch": launch_mode,
         "phases_ms": {"learn": statistics.mean(learn_ms), "solve": statistics.mean(solve_ms),
                       "encode": statistics.mean(enc_ms)},
         "step_stats_ms": {"mean": statistics.mean(each_ms), "median": statistics.median(each_ms),
@@ -970,7 +970,8 @@ def run_reference(args):
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded planted affine maps)",
-           "config": describe(args.config, wl),
+           "config": dict(describe(args.config, wl),
+                         parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": threads, "kind": "oracle", "sample": sample,
                             "cpu_model": cpu_model()},
            "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
