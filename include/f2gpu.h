@@ -323,6 +323,14 @@ enum f2_option {
     F2_OPT_LONG_CALL_ROWS = 15,  /* f2_learn_batched calls of at least this many rows eliminate the contexts
                                     of 4..9 words in CTAs of four warps instead of eight (more contexts
                                     side by side; the longest contexts take longer); default 2^25 */
+    F2_OPT_HANDOFF_REPS = 16,    /* a context owned by a whole CTA whose rank has stopped growing hands
+                                    the rest of its call off to a parallel check when at least this many
+                                    of its representatives are left (a representative outside the basis
+                                    sends the rest back to elimination from there); only in calls of at
+                                    least 16x this many rows; default 0 = never. It pays only where a
+                                    few long contexts bound the call: 8192 took a 10,000-context
+                                    wide-feature learn from 1.61 to 1.56 ms, but the 77,926- and
+                                    4,096-context learns 1-7% longer */
 };
 int f2_set_option(f2_store* store, int option, int64_t value);
 

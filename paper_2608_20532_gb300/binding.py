@@ -43,6 +43,7 @@ F2_OPT_SMALL_BASIS_BYTES = 12
 F2_OPT_DEDUP_SHARDS = 13
 F2_OPT_ENCODE_DIRECT_MAX = 14
 F2_OPT_LONG_CALL_ROWS = 15
+F2_OPT_HANDOFF_REPS = 16
 
 # every entry point of include/f2gpu.h
 EXPORTS = (

@@ -34,6 +34,7 @@ constexpr int DEFAULT_WARP_REGION_BYTES = 12288;  // shared memory of one warp-o
 constexpr int DEFAULT_SMALL_REGION_BYTES = 4096;  // the same in the small-width kernel (d <= 96)
 constexpr int64_t DEFAULT_ENCODE_DIRECT_MAX = 65536;  // encode passes this small skip the grouping
 constexpr int64_t DEFAULT_LONG_CALL_ROWS = int64_t(1) << 25;  // learn calls this long: 4-warp CTAs (4..9 words)
+constexpr int64_t DEFAULT_HANDOFF_REPS = 0;  // representatives left for a saturated context to hand off (0: never)
 constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context gets a whole CTA (at most)
 constexpr int HEAVY_ROWS_MIN = 1024;              // ... and at least, when it scales with the batch:
 constexpr int HEAVY_ROWS_BATCH_DIV = 20000;       // batch rows / this (no duplicate pass), or
@@ -70,7 +71,8 @@ enum Class {
     CLS_DDW_QUAD = 10,
     CLS_DDW_WARP = 11,
     CLS_WIDE_M = 12,   // elimination of rows of 10..17 words (a narrower instance of the wide kernel)
-    NUM_CLASSES = 13
+    CLS_RESUME = 13,   // handed-off contexts sent back by the check (their queue head only)
+    NUM_CLASSES = 14
 };
 static_assert(NUM_CLASSES <= CNT_BEGIN - CNT_HEAD, "counter blocks hold one entry per class");
 constexpr int SMALL_WD = 3;
@@ -355,6 +357,10 @@ struct f2_store {
     int dd_shards;              // most CTAs one context's duplicate pass is split over
     int64_t enc_direct_max;     // encode passes of at most this many queries skip the grouping
     int64_t long_call_rows;     // learn calls of at least this many rows: 4-warp CTAs for 4..9-word contexts
+    int64_t handoff_min;        // representatives left for a saturated context to hand off (0: never)
+    int* hand;                  // hand-off lists: counts [2], snap list/start [2C], resume list/from [2C], chunk counters [2C]
+    uint4* check_rec;           // the check's chunk records (2 x uint4 each), grown per call
+    int64_t check_rec_cap;
     f2::Widths widths;      // width classes of the contexts (computed on first use)
     // second stream of the learn launches (kernels of independent width
     // classes run side by side), its fork and join events; created on first use
@@ -459,14 +465,18 @@ struct F2FillList {
     unsigned long long bytes[MAX];
     unsigned int value[MAX];  // byte value
     int n = 0;
+    bool overflow = false;  // more than MAX ranges: f2_fill refuses the list
     void add(void* ptr, size_t nbytes, unsigned int byte = 0)
     {
-        if (ptr && nbytes && n < MAX) {
-            p[n] = ptr;
-            bytes[n] = nbytes;
-            value[n] = byte & 0xffu;
-            ++n;
+        if (!ptr || !nbytes) return;
+        if (n == MAX) {
+            overflow = true;
+            return;
         }
+        p[n] = ptr;
+        bytes[n] = nbytes;
+        value[n] = byte & 0xffu;
+        ++n;
     }
 };
 cudaError_t f2_fill(const F2FillList& L, cudaStream_t cs);

@@ -46,6 +46,37 @@ using namespace f2;
 
 namespace {
 
+// ---------------------------------------------------------------------------
+// Check of a handed-off context (Sec. 2.2 steps (1)-(3) with the basis
+// fixed).  Its basis stopped growing, so every later representative whose
+// features lie in the span is classified against that basis exactly as the
+// sequential algorithm would (the snapshot argument of the design notes):
+// CTAs claim chunks of CHECK_CHUNK representatives, hold the basis in
+// shared memory (a slot per pivot column) and reduce each representative by
+// the pivot rows its own bits select.  A representative outside the span
+// would extend the basis: the chunk records the first such one, and only
+// representatives before the context's first are counted.  The last chunk
+// of a context commits its counts; if some representative was outside the
+// span, the context is listed for resume_kernel from that one on.
+// ---------------------------------------------------------------------------
+struct CheckArgs {
+    const int64_t* row_off;
+    const int64_t* x_off;
+    const uint32_t* x;
+    const uint4* y;
+    const int32_t* rep_list;  // NULL: every row is its own representative
+    const int32_t* rep_dup;
+    const int32_t* rep_count;
+    const int* snap_count;
+    const int32_t* snap_list;
+    const int32_t* snap_start;
+    int* ctr;                 // [C] chunks claimed, [C] chunks done
+    uint4* rec;               // two uint4 per chunk: (first outside, count lo, count hi, -), (first contradiction)
+    int* resume_count;
+    int32_t* resume_list;
+    int32_t* resume_from;
+};
+
 struct LearnArgs {
     const int64_t* row_off;
     const int64_t* x_off;
@@ -66,6 +97,14 @@ struct LearnArgs {
     int tables;                  // reduce against a lookup table of the snapshot where it pays
     int small_region_words;      // shared memory of a warp-owned context of the small-width kernel
     int cta_region_words;        // shared memory of a CTA-owned context (the launch's dynamic size)
+    // a CTA-owned context whose rank has not grown for HANDOFF_QUIET rounds,
+    // with at least handoff_min representatives left, stops and is listed
+    // here: check_snap_kernel checks the rest against its basis in parallel
+    int handoff_min;             // 0 = never
+    int* snap_count;
+    int32_t* snap_list;
+    int32_t* snap_start;         // its first representative left
+    const int32_t* resume_from;  // resume_kernel: the first representative of each listed context
 };
 
 struct DedupArgs {
@@ -1114,6 +1153,17 @@ __device__ __forceinline__ bool reduce_by_table(uint32_t (&xr)[WD], uint4& yr, c
     return nz;
 }
 
+// Hand-off of saturated contexts (see LearnArgs): the quiet rounds before
+// it, the widest basis the check can hold (shared memory words, a slot per
+// coordinate) and its chunks of representatives; the row widths of the two
+// instances of the wide kernel (the 10..17-word one takes part).
+constexpr int HANDOFF_QUIET = 2;
+constexpr int CHECK_BASIS_WORDS = 14336;  // 56 KB
+constexpr int CHECK_CHUNK = 512;
+constexpr int HANDOFF_CALL_FACTOR = 16;  // calls of fewer rows than this many hand-off minimums hand off none
+constexpr int WIDE_WD = 33;    // widest row (d <= 1056)
+constexpr int WIDE_M_WD = 17;  // rows of 10..17 words (d <= 544): half the registers, two CTAs per SM
+
 // One group (a warp, or the whole CTA) streams the representatives of
 // context c through its basis.
 template <int WD, bool CTA>
@@ -1173,7 +1223,8 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     long long first = LLONG_MAX;
     unsigned long long cnt = 0;
     // prefetched round
-    int nk = t;
+    const int k0 = a.resume_from ? a.resume_from[c] : 0;  // the first representative of this launch
+    int nk = k0 + t;
     bool nvalid = nk < R;
     int ni = nvalid ? (reps ? __ldg(reps + nk) : nk) : 0;
     uint32_t nw = (nvalid && dups) ? (uint32_t)__ldg(dups + nk) : 0u;
@@ -1181,8 +1232,10 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     uint4 yn;
     load_raw<WD>(xc + (int64_t)ni * cd.xw, yc + ni, nvalid, cd.n, cd.xw, xn, yn);
     int stop_at = -1;
+    int snap_at = -1;  // handed off from this representative on
+    int quiet = 0;     // rounds in a row that inserted nothing
     int parity = 0;
-    for (int base = 0; base < R; base += nt, parity ^= 1) {
+    for (int base = k0; base < R; base += nt, parity ^= 1) {
         const bool valid = nvalid;
         const int i = ni;
         const uint32_t weight = 1u + nw;
@@ -1284,6 +1337,16 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
                 }
             }
         }
+        if constexpr (CTA && (WD <= NARROW_WD || WD == WIDE_M_WD)) {
+            // every rank >= 1 saturated context with many representatives
+            // left: hand the rest off to the parallel check (block-uniform)
+            quiet = wmask ? 0 : quiet + 1;
+            if (a.handoff_min > 0 && !a.resume_from && quiet >= HANDOFF_QUIET && R - (base + nt) >= a.handoff_min &&
+                *rank_s < cd.d && cd.d * row_stride(WD) <= CHECK_BASIS_WORDS) {
+                snap_at = base + nt;
+                break;
+            }
+        }
         (void)contra_lane;
     }
     warp_stats(first, cnt);
@@ -1297,7 +1360,10 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
     if (t == 0) {
         s.rank[c] = *rank_s;
         commit_stats(s, c, *first_s, *cnt_s);
-        if (stop_at < 0) {
+        if (snap_at >= 0) {  // rows_seen is advanced by check_snap_kernel (or resume_kernel)
+            a.snap_start[c] = snap_at;
+            a.snap_list[atomicAdd(a.snap_count, 1)] = c;
+        } else if (stop_at < 0) {
             s.rows_seen[c] = seen + T;
         } else {  // rows_seen is advanced by verify_full_kernel
             a.late_start[c] = stop_at;
@@ -1305,6 +1371,182 @@ __device__ void elim_ctx(const StoreDev& s, const LearnArgs& a, int c, uint32_t*
         }
     }
     group_sync<CTA>();
+}
+
+__device__ __forceinline__ int64_t check_slot(const CheckArgs& a, int c)
+{
+    return a.row_off[c] / CHECK_CHUNK + c;  // the context's first chunk record (chunks never overlap)
+}
+
+template <int WD>
+__device__ void check_chunk(const StoreDev& s, const CheckArgs& a, int c, int kb, int ke, const uint32_t* S,
+                            const uint32_t (&P)[WD], uint8_t* flags)
+{
+    const CtxDesc cd = s.desc[c];
+    const int64_t r0 = a.row_off[c];
+    const int32_t* reps = a.rep_list ? a.rep_list + r0 : nullptr;
+    const uint32_t* xc = a.x + a.x_off[c];
+    const uint4* yc = a.y + r0;
+    const uint64_t mixed = mixed_words<WD>(P, cd.d, cd.wd);
+    // every lane of a warp in each round: the pivot walk is warp-uniform
+    for (int base = kb; base < ke; base += blockDim.x) {
+        const int k = base + (int)threadIdx.x;
+        const bool valid = k < ke;
+        const int i = valid ? (reps ? __ldg(reps + k) : k) : 0;
+        uint32_t xin[WD], q[WD];
+        uint4 yr;
+        load_raw<WD>(xc + (int64_t)i * cd.xw, yc + i, valid, cd.n, cd.xw, xin, yr);
+        make_q<WD>(xin, valid, s.raw, q);
+        reduce_snapshot<WD>(q, yr, S, P, mixed);
+        uint32_t resid = 0;
+#pragma unroll
+        for (int w = 0; w < WD; ++w) resid |= q[w] & ~P[w];
+        // 2: outside the span, 1: a contradiction, 0: redundant
+        if (valid) flags[k - kb] = resid ? 2 : (nonzero4(yr) ? 1 : 0);
+    }
+}
+
+// Shared memory of the check: the basis (a slot of row_stride words per
+// column), the chunk's classes (CHECK_CHUNK bytes), then CHECK_CTL_WORDS of
+// control (the pivot words, the claimed chunk, the chunk's sums).
+constexpr int CHECK_CTL_WORDS = 64;
+constexpr int CHECK_SMEM_BYTES = 4 * CHECK_BASIS_WORDS + CHECK_CHUNK + 4 * CHECK_CTL_WORDS;
+
+__global__ void __launch_bounds__(256) check_snap_kernel(StoreDev s, CheckArgs a)
+{
+    extern __shared__ __align__(16) uint32_t smem[];
+    uint32_t* const S = smem;
+    uint8_t* const flags = reinterpret_cast<uint8_t*>(smem + CHECK_BASIS_WORDS);
+    uint32_t* const ctl = smem + CHECK_BASIS_WORDS + CHECK_CHUNK / 4;
+    uint32_t* const Ps = ctl;  // 48 pivot words
+    int* const s_c = reinterpret_cast<int*>(ctl + 48);
+    int* const s_k = s_c + 1;
+    int* const s_first_out = s_c + 2;
+    unsigned long long* const s_cnt = reinterpret_cast<unsigned long long*>(ctl + 52);
+    long long* const s_first = reinterpret_cast<long long*>(ctl + 54);
+    const int t = threadIdx.x;
+    int q = 0, built = -1;
+    for (;;) {
+        if (t == 0) {  // the next chunk, contexts in list order
+            int c = -1, k = 0;
+            const int nq = *a.snap_count;
+            for (; q < nq; ++q) {
+                const int cq = a.snap_list[q];
+                const int R = a.rep_list ? a.rep_count[cq] : (int)(a.row_off[cq + 1] - a.row_off[cq]);
+                k = atomicAdd(a.ctr + cq, 1);
+                if (a.snap_start[cq] + k * CHECK_CHUNK < R) {
+                    c = cq;
+                    break;
+                }
+            }
+            *s_c = c;
+            *s_k = k;
+            *s_first_out = INT_MAX;
+            *s_cnt = 0ull;
+            *s_first = LLONG_MAX;
+        }
+        __syncthreads();
+        const int c = *s_c;
+        const int ck = *s_k;
+        if (c < 0) break;
+        const CtxDesc cd = s.desc[c];
+        const int R = a.rep_list ? a.rep_count[c] : (int)(a.row_off[c + 1] - a.row_off[c]);
+        const int st0 = a.snap_start[c];
+        const int kb = st0 + ck * CHECK_CHUNK;
+        const int ke = (kb + CHECK_CHUNK < R) ? kb + CHECK_CHUNK : R;
+        if (built != c) {  // the basis into shared memory (pivot rows only)
+            if (t < 48) Ps[t] = (t < cd.wd) ? s.pivot[cd.pw_off + t] : 0u;
+            __syncthreads();
+            // the stride of the instance that checks it (rows of 10..17 words: the 17-word one)
+            const int rs = row_stride(cd.wd <= NARROW_WD ? cd.wd : WIDE_M_WD);
+            for (int kk = t; kk < cd.d; kk += blockDim.x) {
+                if (!((Ps[kk >> 5] >> (kk & 31)) & 1u)) continue;
+                uint32_t* row = S + kk * rs;
+                *reinterpret_cast<uint4*>(row) = s.bz[cd.slot_off + kk];
+                const uint32_t* src = s.bx + cd.xw_off + (int64_t)kk * cd.wd;
+                for (int v = 0; v < rs - 4; ++v) row[4 + v] = (v < cd.wd) ? src[v] : 0u;
+            }
+            built = c;
+            __syncthreads();
+        }
+#define F2_CHECK(W)                                                   \
+    {                                                                 \
+        uint32_t P[W];                                                \
+        for (int v = 0; v < W; ++v) P[v] = Ps[v];                     \
+        check_chunk<W>(s, a, c, kb, ke, S, P, flags);                 \
+    }
+        switch (cd.wd) {
+        case 1: F2_CHECK(1); break;
+        case 2: F2_CHECK(2); break;
+        case 3: F2_CHECK(3); break;
+        case 4: F2_CHECK(4); break;
+        case 5: F2_CHECK(5); break;
+        case 6: F2_CHECK(6); break;
+        case 7: F2_CHECK(7); break;
+        case 8: F2_CHECK(8); break;
+        case 9: F2_CHECK(9); break;
+        default: F2_CHECK(WIDE_M_WD); break;
+        }
+#undef F2_CHECK
+        __syncthreads();
+        // the first representative outside the span, then the contradictions
+        // before it (weights: the representative and its repeats)
+        for (int j = t; j < ke - kb; j += blockDim.x)
+            if (flags[j] == 2) atomicMin(s_first_out, kb + j);
+        __syncthreads();
+        const int fo = *s_first_out;
+        unsigned long long cnt = 0;
+        long long first = LLONG_MAX;
+        for (int j = t; j < ke - kb && kb + j < fo; j += blockDim.x) {
+            if (flags[j] != 1) continue;
+            const int k = kb + j;
+            const int i = a.rep_list ? __ldg(a.rep_list + a.row_off[c] + k) : k;
+            cnt += 1u + (a.rep_dup ? (uint32_t)__ldg(a.rep_dup + a.row_off[c] + k) : 0u);
+            first = min(first, (long long)i);
+        }
+        if (cnt) {
+            atomicAdd(s_cnt, cnt);
+            atomicMin(s_first, first);
+        }
+        __syncthreads();
+        if (t == 0) {
+            const int64_t slot = check_slot(a, c) + ck;
+            const unsigned long long sc = *s_cnt;
+            const long long sf = *s_first;
+            a.rec[2 * slot] = make_uint4((uint32_t)fo, (uint32_t)sc, (uint32_t)(sc >> 32), 0u);
+            a.rec[2 * slot + 1] = make_uint4((uint32_t)sf, (uint32_t)((unsigned long long)sf >> 32), 0u, 0u);
+            __threadfence();
+            const int nch = (R - st0 + CHECK_CHUNK - 1) / CHECK_CHUNK;
+            if (atomicAdd(a.ctr + s.num_ctx + c, 1) == nch - 1) {  // the context's last chunk
+                __threadfence();
+                const int64_t s0 = check_slot(a, c);
+                int f = INT_MAX;
+                for (int k = 0; k < nch; ++k) f = min(f, (int)__ldcg(a.rec + 2 * (s0 + k)).x);
+                unsigned long long tot = 0;
+                long long fi = LLONG_MAX;
+                for (int k = 0; k < nch; ++k) {
+                    if (st0 + k * CHECK_CHUNK >= f) break;  // chunks past the first outside
+                    const uint4 r = __ldcg(a.rec + 2 * (s0 + k));
+                    const uint4 r2 = __ldcg(a.rec + 2 * (s0 + k) + 1);
+                    tot += (unsigned long long)r.y | ((unsigned long long)r.z << 32);
+                    fi = min(fi, (long long)((unsigned long long)r2.x | ((unsigned long long)r2.y << 32)));
+                }
+                const long long seen = s.rows_seen[c];
+                if (tot) {
+                    s.n_contra[c] += tot;
+                    s.contra[c] = 1;
+                    if (s.first_contra[c] < 0) s.first_contra[c] = seen + fi;
+                }
+                if (f == INT_MAX) {
+                    s.rows_seen[c] = seen + (a.row_off[c + 1] - a.row_off[c]);
+                } else {  // the rest from the first representative outside the span
+                    a.resume_from[c] = f;
+                    a.resume_list[atomicAdd(a.resume_count, 1)] = c;
+                }
+            }
+        }
+        __syncthreads();
+    }
 }
 
 // Narrow elimination: CTA-owned contexts first (longest first), then
@@ -1373,8 +1615,6 @@ __global__ void __launch_bounds__(NW * 32, SMALL ? 3 : 16 / NW) elim_narrow_kern
     }
 }
 
-constexpr int WIDE_WD = 33;    // widest row (d <= 1056)
-constexpr int WIDE_M_WD = 17;  // rows of 10..17 words (d <= 544): half the registers, two CTAs per SM
 
 // Wide elimination: every context by a whole CTA, rows of up to WDT words.
 template <int WDT, int CLS>
@@ -1905,6 +2145,40 @@ __global__ void __launch_bounds__(FULL_THREADS) verify_full_kernel(StoreDev s, F
     }
 }
 
+// The contexts the check sent back: eliminated in stream order from their
+// first representative outside the snapshot (no further hand-off), one CTA
+// each.  Every width that can hand off has an instance here.
+__global__ void __launch_bounds__(LEARN_WARPS * 32, 1) resume_kernel(StoreDev s, LearnArgs a, const int* resume_count,
+                                                                     const int32_t* resume_list)
+{
+    extern __shared__ __align__(16) uint32_t smem[];
+    __shared__ int s_item;
+    const int n = *resume_count;
+    for (;;) {
+        __syncthreads();
+        if (threadIdx.x == 0) s_item = atomicAdd(a.counters + CNT_HEAD + CLS_RESUME, 1);
+        __syncthreads();
+        const int item = s_item;
+        if (item >= n) break;
+        const int c = resume_list[item];
+        const int wd = s.desc[c].wd;
+#define F2_CALL_RESUME(W) elim_ctx<W, true>(s, a, c, smem, a.cta_region_words)
+        switch (wd) {
+        case 1: F2_CALL_RESUME(1); break;
+        case 2: F2_CALL_RESUME(2); break;
+        case 3: F2_CALL_RESUME(3); break;
+        case 4: F2_CALL_RESUME(4); break;
+        case 5: F2_CALL_RESUME(5); break;
+        case 6: F2_CALL_RESUME(6); break;
+        case 7: F2_CALL_RESUME(7); break;
+        case 8: F2_CALL_RESUME(8); break;
+        case 9: F2_CALL_RESUME(9); break;
+        default: F2_CALL_RESUME(WIDE_M_WD); break;
+        }
+#undef F2_CALL_RESUME
+    }
+}
+
 // Which elimination kernels a store needs, and their widest bases.
 
 size_t narrow_smem(int max_narrow_words, int warp_region_words, int nw)
@@ -1951,7 +2225,7 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
                        int64_t warp_work, int32_t* queue, int32_t* keybuf, int* hist, int num_sms,
                        const Widths& wv, int* full_ctr, unsigned long long* full_cnt,
                        unsigned long long* full_first, cudaStream_t cs, Fork* fk = nullptr, int scale = 0,
-                       bool prezeroed = false, int64_t long_rows = LONG_CALL_ROWS)
+                       bool prezeroed = false, int64_t long_rows = LONG_CALL_ROWS, const CheckArgs* check = nullptr)
 {
     // prezeroed: the caller has cleared full_ctr's first 2C words and late
     // count, full_cnt, full_first (to -1) and hist
@@ -2051,6 +2325,30 @@ int launch_elimination(const StoreDev& sd, const LearnArgs& la, const int64_t* r
     }
     e = f.join();
     if (e != cudaSuccess) return f2_cuda_status(e);
+    if (check && la.handoff_min > 0) {
+        // the handed-off contexts: their remaining representatives checked
+        // in parallel, then any that met a representative outside the
+        // span eliminated from there on
+        const size_t csmem = CHECK_SMEM_BYTES;
+        e = cudaFuncSetAttribute(check_snap_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        check_snap_kernel<<<num_sms * 2, 256, csmem, cs>>>(sd, *check);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        int words = wv.max_small_words > wv.max_narrow_words ? wv.max_small_words : wv.max_narrow_words;
+        if (wv.has_wide_m && elim_words(wv.max_wide_m_d, WIDE_M_WD) > words)
+            words = elim_words(wv.max_wide_m_d, WIDE_M_WD);
+        const size_t rsmem = 4 * (size_t)words;
+        e = cudaFuncSetAttribute(resume_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
+        if (e != cudaSuccess) return f2_cuda_status(e);
+        LearnArgs lr = lx;
+        lr.handoff_min = 0;
+        lr.resume_from = check->resume_from;
+        lr.cta_region_words = words;
+        resume_kernel<<<num_sms, LEARN_WARPS * 32, rsmem, cs>>>(sd, lr, check->resume_count, check->resume_list);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return f2_cuda_status(e);
+    }
     {  // full-rank contexts: at the start of the call (the plan decides on the
        // device which, if any) or reached during it (listed by the kernels above)
         FullArgs fa;
@@ -2134,11 +2432,26 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     }
     // every scratch counter of the call, zeroed by one launch
     const size_t C = (size_t)st->num_ctx;
+    if (st->handoff_min > 0) {  // the check's chunk records, grown stream-ordered
+        const int64_t slots = total_rows / CHECK_CHUNK + (int64_t)C + 1;
+        if (slots > st->check_rec_cap) {
+            if (st->check_rec) cudaFreeAsync(st->check_rec, cs);
+            st->check_rec = nullptr;
+            st->check_rec_cap = 0;
+            if (f2_dev_alloc(st, (void**)&st->check_rec, 2 * sizeof(uint4) * (size_t)slots, cs, true) != cudaSuccess)
+                return F2_ERR_OOM;
+            st->check_rec_cap = slots;
+        }
+    }
     F2FillList zl;
     if (st->timing_on) {  // diagnostics: per-context timestamps of this call
         const size_t bytes = sizeof(unsigned long long) * TIME_WORDS * C;
         if (!st->timing && f2_dev_alloc(st, (void**)&st->timing, bytes, cs, true) != cudaSuccess) return F2_ERR_OOM;
         zl.add(st->timing, bytes);
+    }
+    {  // hand-off: the two list counts and the chunk counters
+        zl.add(st->hand, sizeof(int) * 2);
+        zl.add(st->hand + 2 + 4 * C, sizeof(int) * 2 * C);
     }
     if (dedup) {  // the work totals and the shard items of the duplicate pass
         zl.add(st->counters + CNT_WORK, (CNT_WORDS - CNT_WORK) * sizeof(int));
@@ -2231,6 +2544,13 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     la.tables = st->elim_tables;
     la.small_region_words = (int)(st->small_basis_bytes / 4);
     la.cta_region_words = 0;  // set per launch
+    // hand-off of saturated contexts, in calls long enough to have some
+    la.handoff_min = (st->handoff_min > 0 && total_rows >= HANDOFF_CALL_FACTOR * st->handoff_min)
+                         ? (int)st->handoff_min : 0;
+    la.snap_count = st->hand;
+    la.snap_list = st->hand + 2;
+    la.snap_start = st->hand + 2 + C;
+    la.resume_from = nullptr;
     if (!st->widths_ready) {  // fixed by the widths: computed once per store
         st->widths = width_summary(st->n_bits.data(), st->num_ctx, (st->flags & F2_FLAG_RAW_FEATURES) != 0);
         st->widths_ready = true;
@@ -2247,10 +2567,26 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
         if (heavy > st->heavy_rows) heavy = st->heavy_rows;
     }
     const int scale = dedup && !st->heavy_rows_set && !st->warp_work_set;
+    CheckArgs ca;
+    ca.row_off = row_off;
+    ca.x_off = x_off;
+    ca.x = x;
+    ca.y = reinterpret_cast<const uint4*>(y);
+    ca.rep_list = la.rep_list;
+    ca.rep_dup = la.rep_dup;
+    ca.rep_count = la.rep_count;
+    ca.snap_count = la.snap_count;
+    ca.snap_list = la.snap_list;
+    ca.snap_start = la.snap_start;
+    ca.resume_count = st->hand + 1;
+    ca.resume_list = st->hand + 2 + 2 * C;
+    ca.resume_from = st->hand + 2 + 3 * C;
+    ca.ctr = st->hand + 2 + 4 * C;
+    ca.rec = st->check_rec;
     return launch_elimination(sd, la, row_off, x_off, total_rows, total_x_words, dedup ? st->rep_count : nullptr,
                               heavy, st->warp_work, st->queue, st->keybuf, st->plan_hist + PLAN_HIST_WORDS,
                               st->num_sms, wv, st->full_ctr, st->full_cnt, st->full_first, cs, &fk, scale, true,
-                              st->long_call_rows);
+                              st->long_call_rows, &ca);
 }
 
 extern "C" int f2_learn_timing(const f2_store* st, uint64_t* out_host, f2_stream_t stream)
@@ -2498,6 +2834,11 @@ extern "C" int f2_learn_batched_noalloc(int32_t num_ctx, const int32_t* n_bits_h
     la.tables = 1;
     la.small_region_words = DEFAULT_SMALL_REGION_BYTES / 4;
     la.cta_region_words = 0;
+    la.handoff_min = 0;
+    la.snap_count = nullptr;
+    la.snap_list = nullptr;
+    la.snap_start = nullptr;
+    la.resume_from = nullptr;
     la.warp_region_words = NOALLOC_WARP_REGION_WORDS;
     const Widths wv = width_summary(n_bits_host, num_ctx, raw);
     return launch_elimination(sd, la, row_off_dev, x_off_dev, total_rows, total_x_words, nullptr, NOALLOC_HEAVY_ROWS,

@@ -57,6 +57,7 @@ __global__ void __launch_bounds__(256) fill_kernel(F2FillList L)
 
 cudaError_t f2_fill(const F2FillList& L, cudaStream_t cs)
 {
+    if (L.overflow) return cudaErrorInvalidValue;
     if (L.n == 0) return cudaSuccess;
     unsigned long long total = 0;
     for (int k = 0; k < L.n; ++k) total += L.bytes[k];
@@ -113,6 +114,7 @@ static void free_store(f2_store* s)
     void* ptrs[] = {s->desc,   s->rank,   s->contra,   s->first_contra, s->n_contra, s->rows_seen,
                     s->pivot,  s->bx,     s->bz,       s->status,       s->queue,    s->keybuf,
                     s->counters, s->plan_hist, s->rep_count, s->rep_list, s->rep_dup, s->shard_reps, s->shard_done,
+                    s->hand, s->check_rec,
                     s->full_ctr, s->full_cnt, s->full_first,
                     s->enc_bins, s->enc_off, s->enc_sorted, s->enc_items, s->enc_hot, s->enc_tab_off,
                     s->enc_pool, s->timing};
@@ -159,6 +161,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     s->dd_shards = 4;
     s->enc_direct_max = DEFAULT_ENCODE_DIRECT_MAX;
     s->long_call_rows = DEFAULT_LONG_CALL_ROWS;
+    s->handoff_min = DEFAULT_HANDOFF_REPS;
     s->enc_table_min = f2_encode_table_min_default();
     s->enc_chunk_shift = f2_encode_chunk_shift_default();
     s->enc_chunk_min = f2_encode_chunk_min_default();
@@ -219,6 +222,7 @@ extern "C" int f2_create(f2_store** out, int32_t num_ctx, const int32_t* n_bits_
     alloc((void**)&s->rep_count, sizeof(int32_t) * C);
     alloc((void**)&s->shard_reps, sizeof(int32_t) * 8 * C);
     alloc((void**)&s->shard_done, sizeof(int32_t) * C);
+    alloc((void**)&s->hand, sizeof(int) * (2 + 6 * C));
     alloc((void**)&s->plan_hist, sizeof(int) * 2 * PLAN_HIST_WORDS);  // the two plans of a learn call
     alloc((void**)&s->full_ctr, sizeof(int) * (4 * C + 1));
     alloc((void**)&s->full_cnt, sizeof(unsigned long long) * C);
@@ -492,6 +496,10 @@ extern "C" int f2_set_option(f2_store* s, int option, int64_t value)
     case F2_OPT_SMALL_BASIS_BYTES:
         if (value < 4096 || value > 24576) return F2_ERR_INVALID_ARG;
         s->small_basis_bytes = (value / 16) * 16;
+        return F2_OK;
+    case F2_OPT_HANDOFF_REPS:
+        if (value < 0 || value > (int64_t(1) << 30)) return F2_ERR_INVALID_ARG;
+        s->handoff_min = value;
         return F2_OK;
     case F2_OPT_LONG_CALL_ROWS:
         if (value < 0) return F2_ERR_INVALID_ARG;

@@ -184,6 +184,70 @@ def test_dedup_shards(env, shards):
     _check_store(binding, st, O, queries=(q.ctx_id, q.x))
 
 
+def _affine_rows(rng, n, T, r1, late_new, contra_at):
+    """T observations of one context: x in the span of r1 random generators
+    (two more from row 0.8 T on when late_new), half of them repeats of
+    earlier rows, y a planted affine map of x, and the rows in contra_at
+    repeats of earlier rows with one flipped word bit (contradictions)."""
+    W = (n + 31) // 32
+    def rand_vec(k):
+        v = rng.integers(0, 2 ** 32, size=(k, W), dtype=np.uint64).astype(np.uint32)
+        if n % 32:
+            v[:, -1] &= np.uint32((1 << (n % 32)) - 1)
+        return v
+    gens, late = rand_vec(r1), rand_vec(2)
+    coef = rng.random((T, r1)) < 0.5
+    x = np.zeros((T, W), np.uint32)
+    for j in range(r1):
+        x ^= gens[j] * coef[:, j:j + 1].astype(np.uint32)
+    if late_new:
+        lo = int(0.8 * T)
+        for j in range(2):
+            x[lo:] ^= late[j] * (rng.random((T - lo, 1)) < 0.5).astype(np.uint32)
+    cols = rng.integers(0, 2 ** 32, size=(n + 1, 4), dtype=np.uint64).astype(np.uint32)
+    def word(xr):
+        yv = cols[0].copy()
+        for j in range(n):
+            if (int(xr[j // 32]) >> (j % 32)) & 1:
+                yv ^= cols[1 + j]
+        return yv
+    y = np.stack([word(x[i]) for i in range(T)])
+    for i in range(1, T):  # repeats of earlier rows
+        if rng.random() < 0.5:
+            k = int(rng.integers(0, i))
+            x[i], y[i] = x[k], y[k]
+    for i in contra_at:
+        k = int(rng.integers(0, i))
+        x[i], y[i] = x[k], y[k].copy()
+        y[i][0] ^= np.uint32(1)
+    return [(x[i], y[i]) for i in range(T)]
+
+
+@pytest.mark.parametrize("late_new", [False, True])
+def test_handoff_check_and_resume(env, late_new):
+    """A CTA-owned context whose rank stops growing hands the rest of its
+    rows off to the parallel check (F2_OPT_HANDOFF_REPS); with late_new a
+    row outside the basis turns up there and sends the rest back to
+    elimination from that row.  Contradictions before and after that point;
+    every exported array and the solve equal the oracle's."""
+    binding, dev = env
+    rng = np.random.default_rng(4242 + int(late_new))
+    n_bits = [20, 40, 70, 100, 150, 260, 400]
+    T = 3000
+    systems = [_affine_rows(rng, n, T, int(rng.integers(3, 12)), late_new, [900, 2700]) for n in n_bits]
+    ro, xo, x, y = csr_from_rows(n_bits, systems)
+    for opts in ({binding.F2_OPT_HEAVY_ROWS: 1, binding.F2_OPT_HANDOFF_REPS: 256},
+                 {binding.F2_OPT_HEAVY_ROWS: 1, binding.F2_OPT_HANDOFF_REPS: 256, binding.F2_OPT_DEDUP: 0},
+                 {binding.F2_OPT_HEAVY_ROWS: 1, binding.F2_OPT_HANDOFF_REPS: 0}):
+        st = _learn_csr(binding, dev, n_bits, ro, xo, x, y, options=opts)
+        O = oracle.Oracle(n_bits, threads=2)
+        O.learn(ro, xo, x, y)
+        _check_store(binding, st, O)
+        ex = O.export()
+        assert ex["contra"].all()  # both planted contradictions in every context
+        st.close()
+
+
 def test_config3_scaled(env):
     binding, dev = env
     wl = wlmod.generate(wlmod.scaled(3, 1500), 303, query_count=50000)
