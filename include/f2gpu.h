@@ -285,7 +285,8 @@ enum f2_option {
     F2_OPT_HEAVY_ROWS = 1,   /* contexts with at least this many rows in a call get a whole CTA; unless
                                 this or F2_OPT_WARP_WORK is set, the call scales both to its own work
                                 (representatives / (20 SMs), within [1024, 4096]; with the duplicate
-                                pass off, rows / 20000) */
+                                pass off, rows / 20000). Unless this is set, a store of at most two
+                                contexts per SM gives every context a whole CTA */
     F2_OPT_WARP_BASIS_BYTES = 2, /* shared memory (bytes) of one warp-owned context */
     F2_OPT_WARP_WORK = 3,        /* largest rows x d (per call) of a warp-owned context; default 131072,
                                     scaled like F2_OPT_HEAVY_ROWS (sum of rows x d / (45 SMs), at least

@@ -39,6 +39,7 @@ constexpr int DEFAULT_HEAVY_ROWS = 4096;          // rows from which a context g
 constexpr int HEAVY_ROWS_MIN = 1024;              // ... and at least, when it scales with the batch:
 constexpr int HEAVY_ROWS_BATCH_DIV = 20000;       // batch rows / this (no duplicate pass), or
 constexpr int HEAVY_REPS_DIV = 20;                // representatives / (SMs x this) after the duplicate pass
+constexpr int ALL_CTA_PER_SM = 2;                 // stores of at most this many contexts per SM: a CTA each
 constexpr long long WARP_WORK_MIN = 32768;        // scaled warp work (rows x d) stays within
 constexpr int WARP_WORK_DIV = 45;                 // [this, the option]: sum(rows x d) / (SMs x this)
 constexpr long long DEFAULT_WARP_WORK = 131072;   // largest rows x d handled by one warp

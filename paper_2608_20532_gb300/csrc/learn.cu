@@ -2560,13 +2560,19 @@ extern "C" int f2_learn_batched(f2_store* st, const int64_t* row_off, const uint
     // scales with the batch -- in a short call a warp-owned context of a few
     // thousand rows, dependent round after round, would outlast everything
     // else, while in a long one warps keep the SMs fuller
+    // else, and in a store of at most ALL_CTA_PER_SM contexts per SM, every
+    // context gets one: none waits for a CTA, and a CTA takes eight warps'
+    // rows per dependent round
     int64_t heavy = st->heavy_rows;
-    if (!st->heavy_rows_set && !dedup) {
+    const bool all_cta = !st->heavy_rows_set && st->num_ctx <= (int64_t)ALL_CTA_PER_SM * st->num_sms;
+    if (all_cta) {
+        heavy = 1;
+    } else if (!st->heavy_rows_set && !dedup) {
         heavy = total_rows / HEAVY_ROWS_BATCH_DIV;
         if (heavy < HEAVY_ROWS_MIN) heavy = HEAVY_ROWS_MIN;
         if (heavy > st->heavy_rows) heavy = st->heavy_rows;
     }
-    const int scale = dedup && !st->heavy_rows_set && !st->warp_work_set;
+    const int scale = dedup && !all_cta && !st->heavy_rows_set && !st->warp_work_set;
     CheckArgs ca;
     ca.row_off = row_off;
     ca.x_off = x_off;

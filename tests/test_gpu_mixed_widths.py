@@ -52,8 +52,9 @@ def test_every_width_class_in_one_store(host, all_cta):
     binding = lib()
     n_bits, batches = _mixed(11)
     st = binding.Store(n_bits, device=dev)
-    if all_cta:  # every context eliminated by a whole CTA
-        st.set_option(binding.F2_OPT_HEAVY_ROWS, 1)
+    # all_cta: every context eliminated by a whole CTA (a store of 57 contexts
+    # is that by default); else warps own every context whose basis fits
+    st.set_option(binding.F2_OPT_HEAVY_ROWS, 1 if all_cta else 1 << 40)
     if host:
         st.set_option(binding.F2_OPT_HOST_CHUNK_BYTES, 1 << 16)
     O = oracle.Oracle(n_bits, threads=4)

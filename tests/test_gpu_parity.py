@@ -127,7 +127,8 @@ def test_tiny_random_systems(env, seed, mode):
     binding, dev = env
     ds, systems = _random_tiny(seed)
     ro, xo, x, y = csr_from_rows(ds, systems)
-    opts = {binding.F2_OPT_HEAVY_ROWS: 1} if mode == "cta" else {}
+    # a store this small gives every context a CTA unless the threshold is set
+    opts = {binding.F2_OPT_HEAVY_ROWS: 1 if mode == "cta" else 1 << 40}
     st = _learn_csr(binding, dev, ds, ro, xo, x, y, raw=True, options=opts)
     O = oracle.Oracle(ds, raw=True, threads=1)
     O.learn(ro, xo, x, y)
@@ -278,7 +279,7 @@ def test_width_boundaries(env, n):
     cfg = dict(num_ctx=5, layout=wlmod.LAYOUT_UNIFORM_BITS, n_fixed=n, rows_fixed=max(8, min(3 * n, 1500)),
                dup_frac=0.0, density=0.3, n_contra=2)
     wl = wlmod.generate(cfg, 1000 + n)
-    for opts in ({}, {binding.F2_OPT_HEAVY_ROWS: 1}):
+    for opts in ({}, {binding.F2_OPT_HEAVY_ROWS: 1 << 40}):  # (five contexts: a CTA each by default)
         st = binding.Store(wl.n_bits, device=dev)
         for k, v in opts.items():
             st.set_option(k, v)
@@ -308,7 +309,7 @@ def test_edge_cases(env):
         [(np.array([7], np.uint32), y1), (np.array([15], np.uint32), y1 ^ np.array([1, 0, 0, 0], np.uint32))],  # bits above n ignored
     ]
     ro, xo, x, y = csr_from_rows(n_bits, rows)
-    for opts in ({}, {binding.F2_OPT_HEAVY_ROWS: 1}):
+    for opts in ({}, {binding.F2_OPT_HEAVY_ROWS: 1 << 40}):  # (six contexts: a CTA each by default)
         st = _learn_csr(binding, dev, n_bits, ro, xo, x, y, options=opts)
         O = oracle.Oracle(n_bits, threads=1)
         O.learn(ro, xo, x, y)
