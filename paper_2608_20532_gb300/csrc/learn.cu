@@ -48,16 +48,17 @@ namespace {
 
 // ---------------------------------------------------------------------------
 // Check of a handed-off context (Sec. 2.2 steps (1)-(3) with the basis
-// fixed).  Its basis stopped growing, so every later representative whose
-// features lie in the span is classified against that basis exactly as the
-// sequential algorithm would (the snapshot argument of the design notes):
-// CTAs claim chunks of CHECK_CHUNK representatives, hold the basis in
-// shared memory (a slot per pivot column) and reduce each representative by
-// the pivot rows its own bits select.  A representative outside the span
-// would extend the basis: the chunk records the first such one, and only
-// representatives before the context's first are counted.  The last chunk
-// of a context commits its counts; if some representative was outside the
-// span, the context is listed for resume_kernel from that one on.
+// fixed).  Until a representative falls outside the span, the sequential
+// algorithm leaves the basis as it is, so it classifies every such
+// representative against this basis, and in any order: CTAs claim chunks
+// of CHECK_CHUNK representatives, hold the basis in shared memory (a slot
+// per pivot column) and reduce each representative by the pivot rows its
+// own bits select (the warp walks the pivots set in any of its lanes).  A
+// representative outside the span would extend the basis: the chunk
+// records the first such one, and only representatives before the
+// context's first are counted.  The last chunk of a context commits its
+// counts; if some representative was outside the span, the context is
+// listed for resume_kernel from that one on.
 // ---------------------------------------------------------------------------
 struct CheckArgs {
     const int64_t* row_off;
