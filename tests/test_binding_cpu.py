@@ -61,3 +61,33 @@ def test_missing_library_fails_loudly(tmp_path):
 
     with pytest.raises(RuntimeError):
         binding.load_library(str(tmp_path / "nope.so"))
+
+
+def _header_constants():
+    """Every F2_* enumerator and numeric #define of the headers, by value."""
+    consts = {}
+    inc = os.path.join(ROOT, "include")
+    for h in sorted(os.listdir(inc)):
+        if not h.endswith(".h"):
+            continue
+        with open(os.path.join(inc, h)) as f:
+            text = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
+        for name, val in re.findall(r"\b(F2_[A-Z0-9_]+)\s*=\s*(-?\d+)", text):
+            consts[name] = int(val)
+        for name, val in re.findall(r"#define\s+(F2_[A-Z0-9_]+)\s+(\d+)u?\b", text):
+            consts[name] = int(val)
+    return consts
+
+
+def test_binding_constants_match_the_header():
+    """The binding's status codes, flags and option numbers are the header's."""
+    from paper_2608_20532_gb300 import binding
+
+    consts = _header_constants()
+    for prefix in ("F2_OK", "F2_ERR_", "F2_FLAG_", "F2_OPT_"):
+        names = [n for n in consts if n.startswith(prefix)]
+        assert names, prefix
+        for n in names:
+            assert getattr(binding, n, None) == consts[n], n
+    ours = [n for n in dir(binding) if n.startswith(("F2_OPT_", "F2_ERR_", "F2_FLAG_"))]
+    assert set(ours) <= set(consts), set(ours) - set(consts)
